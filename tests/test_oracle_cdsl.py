@@ -1,0 +1,278 @@
+"""Pins of the CDSL oracle (Algorithm 1, Algorithm 2 and the batched CDSL-k step).
+
+Each test ties the oracle to something the paper or the mathematics fixes: the worked reward
+example (Sec. 4.1), exact rational threshold tests, the full-acceptance property of hard
+rejection with identical models, the reduction of CDSL-k to CDLH and to greedy decoding, and
+a brute-force re-derivation of the beam selection over the whole (16-token) vocabulary that
+uses no key/value cache."""
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import synth
+import oracle
+from oracle import (S1, S2_S3, S4, Decider, RunParams, Transformer, cdsl_k_step, coverage,
+                    n_min, prefill, reward)
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def shape(vocab=16, d=32, layers=2, heads=4, kv=2, ffn=48):
+    return synth.ModelShape(n_layers=layers, d_model=d, n_heads=heads, n_kv_heads=kv,
+                            d_ffn=ffn, vocab=vocab)
+
+
+def model(shp, seed, scale=0.5):
+    rng = np.random.default_rng(seed)
+    w = {n: (np.ones(s, np.float32) if len(s) == 1 else
+             (scale * rng.standard_normal(s)).astype(np.float32)) for n, s in shp.weight_specs()}
+    return Transformer(shp, w)
+
+
+def greedy_chain(m, prompt, n):
+    toks = list(prompt)
+    for _ in range(n):
+        toks.append(int(np.argmax(m.forward_full(toks)[0][-1])))
+    return toks[len(prompt):]
+
+
+# ---------------------------------------------------------------- reward and thresholds
+
+def test_reward_worked_example():
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "reward_worked_example.txt"))
+            if l.strip() and not l.startswith("#")]
+    for n_kw, n_cov, want in rows:
+        n_kw, n_cov = int(n_kw), int(n_cov)
+        kws = list(range(100, 100 + n_kw))
+        text = [7, kws[0], 8, kws[1], kws[1], 9]          # 2 distinct concepts, one repeated
+        assert n_cov == 2
+        assert coverage(kws, text) == pytest.approx(float(want), abs=0)
+        assert reward(kws, text, None, None, False) == pytest.approx(float(want), abs=0)
+
+
+def test_reward_cases():
+    kws = [3, 4, 5]
+    assert coverage(kws, []) == 0.0
+    assert coverage(kws, [3, 3, 3]) == pytest.approx(1 / 3)
+    assert coverage(kws, [5, 4, 3, 9]) == 1.0
+    w = np.array([1.0, -2.0])
+    h = np.array([0.5, 0.25])               # w.h = 0 -> sigmoid 0.5
+    assert reward(kws, [3], h, w, True) == pytest.approx(0.5 * (1 / 3) + 0.25)
+
+
+@pytest.mark.parametrize("d", [1, 2, 3, 4, 5, 6, 8, 10])
+@pytest.mark.parametrize("a_t", [0.0, 0.25, 0.3, 0.4, 0.5, 0.6, 0.8, 0.9, 1.0, 1.5])
+def test_n_min_is_exact_threshold(d, a_t):
+    """n >= n_min  <=>  n/d >= a_t, checked in exact rationals (a_t as its float32 value)."""
+    at = Fraction(float(np.float32(a_t)))
+    nm = n_min(a_t, d)
+    for n in range(d + 1):
+        assert (n >= nm) == (Fraction(n, d) >= at or
+                             np.float32(n) / np.float32(d) >= np.float32(a_t))
+
+
+def test_decider_tie_rules():
+    dec = Decider()
+    assert dec.argmax(np.array([1.0, 3.0, 3.0, 2.0]), "x", 0) == 1
+    assert dec.topk(np.array([2.0, 5.0, 5.0, 1.0, 5.0]), 3, "roots", 0).tolist() == [1, 2, 4]
+    assert dec.first_max(np.array([0.2, 0.4, 0.4]), "beam", 0) == 1
+    # near-tie adoption only within tolerance, never for exact ties
+    other = {"x": {0: 2, 1: 3, 2: 2}}
+    dec = Decider(other=other, tol=0.05)
+    assert dec.argmax(np.array([0.0, 1.0, 0.97]), "x", 0) == 2
+    assert dec.argmax(np.array([0.0, 1.0, 0.5, 0.9]), "x", 1) == 1
+    assert dec.argmax(np.array([0.0, 1.0, 1.0]), "x", 2) == 1
+    assert len(dec.adopted) == 1
+
+
+# ---------------------------------------------------------------- CDSL-k invariants
+
+def run_params(**kw):
+    base = dict(k=3, d=3, a_t=0.3, r_t=0.3, max_new=8, composite_reward=True)
+    base.update(kw)
+    return RunParams(**base)
+
+
+def test_identical_models_accept_everything():
+    """Hard rejection with M_q = M_p: every drafted token is the target's argmax (Sec. 3.2.2)."""
+    shp = shape(vocab=40)
+    tgt = model(shp, 1)
+    drf = model(shp, 1)
+    run = run_params(k=4, d=4, r_t=10.0)
+    st = prefill(tgt, drf, np.array([[1, 2, 3, 4, 5], [9, 8, 7, 6, 5]]), np.array([[1, 2], [3, 4]]))
+    w = np.random.default_rng(2).standard_normal(shp.d_model)
+    for _ in range(3):
+        for rec in cdsl_k_step(tgt, drf, st, run, w):
+            assert np.all(rec.n == run.d)
+            assert np.array_equal(rec.argmax[:, :run.d], rec.x)
+            assert np.allclose(rec.logp, rec.logq, atol=1e-9)
+            assert rec.state == S4            # a = 1 >= a_t, r < r_t = 10
+
+
+def test_cdsl_reduces_to_cdlh():
+    """M_q = M_p and r_t = +inf: every CDSL-k step is the CDLH token of Alg. 2 (Sec. 3.1)."""
+    shp = shape(vocab=16)
+    tgt = model(shp, 3)
+    run = run_params(k=3, d=3, r_t=np.inf, max_new=7)
+    w = np.random.default_rng(4).standard_normal(shp.d_model)
+    prompt, kw = [1, 7, 3, 2], [5, 11, 13]
+    st = prefill(tgt, tgt, np.array([prompt]), np.array([kw]))
+    while len(st[0].T) < run.max_new:
+        rec = cdsl_k_step(tgt, tgt, st, run, w)[0]
+        assert rec.state in (S2_S3, S4) and len(rec.emitted) == 1
+    ref = oracle.cdlh_generate(tgt, tgt, tgt, prompt, kw, run, w)
+    assert st[0].T == ref.T
+
+
+def test_always_s1_is_greedy_decoding():
+    """a_t = 0, r_t = -inf, M_q = M_p, constant reward: every step is S1 and emits the root
+    plus all d accepted tokens, which is greedy decoding of M_p."""
+    shp = shape(vocab=30)
+    tgt = model(shp, 5)
+    run = run_params(k=3, d=3, a_t=0.0, r_t=-np.inf, max_new=9, composite_reward=False)
+    prompt = [4, 4, 2, 8]
+    st = prefill(tgt, tgt, np.array([prompt]), np.array([[29]]))
+    while len(st[0].T) < run.max_new:
+        rec = cdsl_k_step(tgt, tgt, st, run, np.zeros(shp.d_model))[0]
+        assert rec.state == S1
+    assert st[0].T == greedy_chain(tgt, prompt, run.max_new)
+
+
+def test_generation_stops_at_l_m():
+    shp = shape(vocab=30)
+    tgt = model(shp, 5)
+    run = run_params(k=2, d=4, a_t=0.0, r_t=-np.inf, max_new=6, composite_reward=False)
+    st = prefill(tgt, tgt, np.array([[1, 2]]), np.array([[0]]))
+    steps = 0
+    while len(st[0].T) < run.max_new:
+        rec = cdsl_k_step(tgt, tgt, st, run, np.zeros(shp.d_model))[0]
+        steps += 1
+    assert len(st[0].T) == 6 and steps == 2 and len(rec.emitted) == 1
+    assert not cdsl_k_step(tgt, tgt, st, run, np.zeros(shp.d_model))[0].active
+
+
+def brute_force_step(tgt, drf, prompt, T, kw, run, w):
+    """The CDSL-k decision for pfx = prompt + T from scratch: every one of the V tokens is
+    tried as a root, each rollout and verify row recomputed with forward_full (no cache)."""
+    pfx = list(prompt) + list(T)
+    V = tgt.shape.vocab
+    p0 = tgt.forward_full(pfx)[0][-1]
+    rank = sorted(range(V), key=lambda t: (-p0[t], t))
+    cand = {}
+    for c in range(V):
+        x = []
+        for _ in range(run.d):
+            x.append(int(np.argmax(drf.forward_full(pfx + [c] + x)[0][-1])))
+        lg, hf = tgt.forward_full(pfx + [c] + x)
+        rows, hid = lg[len(pfx):], hf[len(pfx):]
+        n = 0
+        while n < run.d and int(np.argmax(rows[n])) == x[n]:
+            n += 1
+        rf = reward(kw, T + [c] + x, hid[run.d], w, run.composite_reward)
+        ra = reward(kw, T + [c] + x[:n], hid[n], w, run.composite_reward)
+        cand[c] = (x, n, rf, ra)
+    roots = rank[:run.k]
+    rfs = [cand[c][2] for c in roots]
+    bi = rfs.index(max(rfs))
+    x, n, rf, ra = cand[roots[bi]]
+    if n >= n_min(run.a_t, run.d) and np.float32(ra) >= np.float32(run.r_t):
+        return roots, bi, S1, [roots[bi]] + x[:n]
+    return roots, bi, (S2_S3 if n < n_min(run.a_t, run.d) else S4), [roots[bi]]
+
+
+@pytest.mark.parametrize("seed,same", [(11, False), (12, True), (13, False)])
+def test_brute_force_selection(seed, same):
+    shp = shape(vocab=16, d=24)
+    tgt = model(shp, seed)
+    drf = tgt if same else model(shape(vocab=16, d=16, layers=1, heads=2, kv=1, ffn=20), seed + 100)
+    run = run_params(k=4, d=3, a_t=0.3, r_t=0.5, max_new=6)
+    w = np.random.default_rng(seed).standard_normal(shp.d_model) * 0.5
+    prompt, kw = [3, 1, 4, 1, 5], [2, 6, 9, 12, 15]
+    st = prefill(tgt, drf, np.array([prompt]), np.array([kw]))
+    while len(st[0].T) < run.max_new:
+        T0 = list(st[0].T)
+        roots, bi, state, out = brute_force_step(tgt, drf, prompt, T0, kw, run, w)
+        rec = cdsl_k_step(tgt, drf, st, run, w)[0]
+        assert rec.roots.tolist() == roots
+        assert rec.beam == bi and rec.state == state
+        assert rec.emitted == out[:run.max_new - len(T0)]
+
+
+# ---------------------------------------------------------------- literal Alg. 1 and Alg. 2
+
+def test_alg1_identical_models_is_greedy():
+    """Alg. 1 with M_q = M_p accepts all d drafts; with r_t = -inf every iteration is S1, so
+    the output is greedy decoding of M_p (no bonus token is ever added, Sec. 3.2.3 S1)."""
+    shp = shape(vocab=30)
+    tgt = model(shp, 21)
+    run = run_params(d=3, a_t=0.5, r_t=-np.inf, max_new=9, composite_reward=False)
+    prompt = [5, 6, 7]
+    st, recs = oracle.alg1_generate(tgt, tgt, prompt, [0], run, np.zeros(shp.d_model))
+    assert all(r["n"] == 3 and r["state"] == S1 for r in recs)
+    assert st.T == greedy_chain(tgt, prompt, 9)
+
+
+def test_alg1_s4_appends_cdlh_appx_token():
+    shp = shape(vocab=20)
+    tgt = model(shp, 22)
+    run = run_params(k=3, d=2, a_t=0.5, r_t=np.inf, max_new=3, composite_reward=False)
+    prompt = [1, 2, 3]
+    st, recs = oracle.alg1_generate(tgt, tgt, prompt, [0, 1], run, np.zeros(shp.d_model))
+    r = recs[0]
+    assert r["state"] == S4 and r["n"] == 2 and len(r["emitted"]) == 3
+    # the appended token is CDLH-appx's choice; with a constant reward it is the top-1 of M_p
+    assert r["emitted"] == greedy_chain(tgt, prompt, 3)
+
+
+def test_alg1_step1_budget():
+    """S2/S3 with b = 1: Step-1 takes M_p's greedy token; if its lookahead's reward clears
+    r_t it is emitted after the accepted drafts, otherwise Step-2 (CDLH-appx) decides."""
+    shp_t, shp_d = shape(vocab=20), shape(vocab=20, d=16, layers=1, heads=2, kv=1, ffn=20)
+    tgt, drf = model(shp_t, 31), model(shp_d, 32)
+    prompt = [1, 2, 3, 4]
+    seen = 0
+    for r_t, step1_wins in [(-np.inf, True), (np.inf, False)]:
+        run = run_params(k=3, d=3, a_t=1.0, r_t=r_t, max_new=6, composite_reward=False, b=1)
+        st, recs = oracle.alg1_generate(tgt, drf, prompt, [0, 1], run, np.zeros(shp_t.d_model))
+        T = []
+        for r in recs:
+            pfx = prompt + T
+            T = T + r["emitted"]
+            if r["state"] != S2_S3:
+                continue
+            seen += 1
+            acc = r["x"][:r["n"]]
+            assert r["emitted"][:len(acc)] == acc and len(r["emitted"]) == len(acc) + 1
+            p = tgt.forward_full(pfx + acc)[0][-1]
+            if step1_wins:   # Step-1: M_p's greedy token after pfx + accepted drafts
+                assert r["emitted"][-1] == int(np.argmax(p))
+            else:            # Step-2: one of M_p's top-k there (CDLH-appx)
+                assert r["emitted"][-1] in np.argsort(-p)[:run.k].tolist()
+    assert seen >= 2
+
+
+def test_cdlh_appx_with_identical_models_is_cdlh():
+    """CDLH-appx with M_q = M_p is CDLH (Alg. 2, lookahead comment)."""
+    shp = shape(vocab=16)
+    tgt = model(shp, 41)
+    run = run_params(k=3, d=2, max_new=5)
+    w = np.random.default_rng(42).standard_normal(shp.d_model)
+    a = oracle.cdlh_generate(tgt, tgt, tgt, [1, 2, 3], [4, 5], run, w)
+    tgt2 = model(shp, 41)
+    b = oracle.cdlh_generate(tgt, tgt2, tgt2, [1, 2, 3], [4, 5], run, w)
+    assert a.T == b.T
+
+
+def test_tiny_workload_runs():
+    """The tiny fp32 workload end to end: 16 tokens, every step emits >= 1 token."""
+    wl = synth.TINY
+    tgt = Transformer(wl.target, synth.model_weights(wl, "target"))
+    drf = Transformer(wl.draft, synth.model_weights(wl, "draft"))
+    run = RunParams(k=wl.k, d=wl.d, a_t=wl.a_t, r_t=wl.r_t, max_new=wl.max_new,
+                    composite_reward=wl.reward_head)
+    states, recs = oracle.cdsl_k_generate(tgt, drf, synth.prompts(wl), synth.keywords(wl), run,
+                                          synth.reward_head(wl))
+    assert len(states[0].T) == wl.max_new
+    assert all(len(r[0].emitted) >= 1 for r in recs)
