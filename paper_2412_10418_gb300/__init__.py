@@ -1,0 +1,281 @@
+"""GB300 CDSL lookahead step: Python binding of the C ABI in include/cdsl.h.
+
+Argument marshalling only: every step of the path runs in the CUDA library
+``libcdsl_gb300.so`` (built in-tree by ``paper_2412_10418_gb300.build``). Importing this module
+fails loudly when the library is missing; there is no CPU fallback.
+
+Functions carry the C names (``cdsl_init``, ``cdsl_prefill``, ``cdsl_lookahead``,
+``cdsl_verify``, ``cdsl_select``, ``cdsl_step`` ...) and take torch CUDA tensors where the C
+call takes device pointers. ``Engine`` bundles a context with its workspace and outputs.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import List, Optional, Sequence
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libcdsl_gb300.so")
+
+DTYPE_F32, DTYPE_BF16 = 0, 1
+STATUS = {0: "CDSL_OK", 1: "CDSL_EINVAL", 2: "CDSL_ENOMEM", 3: "CDSL_ECUDA", 4: "CDSL_ETIMEOUT",
+          5: "CDSL_ENONFINITE", 6: "CDSL_ESTATE", 7: "CDSL_ERANGE"}
+S1, S2_S3, S4 = 1, 2, 4
+
+
+class CdslError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"{STATUS.get(code, code)}: {msg}")
+        self.code = code
+
+
+class ModelCfg(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32),
+                ("n_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("d_ffn", ctypes.c_int32),
+                ("vocab", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("rope_theta", ctypes.c_float), ("norm_eps", ctypes.c_float)]
+
+
+class RunCfg(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("k", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("max_prompt", ctypes.c_int32), ("max_new", ctypes.c_int32),
+                ("n_keywords", ctypes.c_int32), ("a_t", ctypes.c_float), ("r_t", ctypes.c_float),
+                ("reward_head", ctypes.c_int32), ("page_size", ctypes.c_int32),
+                ("max_chunk", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int32
+EXPORTS = {
+    "cdsl_num_weights": (_I, [ctypes.POINTER(ModelCfg)]),
+    "cdsl_workspace_size": (_I, [ctypes.POINTER(ModelCfg), ctypes.POINTER(ModelCfg),
+                                 ctypes.POINTER(RunCfg), ctypes.POINTER(ctypes.c_size_t)]),
+    "cdsl_init": (_I, [ctypes.POINTER(ModelCfg), ctypes.POINTER(_P), ctypes.POINTER(ModelCfg),
+                       ctypes.POINTER(_P), ctypes.POINTER(RunCfg), _P, _P, ctypes.c_size_t, _P,
+                       ctypes.POINTER(_P)]),
+    "cdsl_prefill": (_I, [_P, _P, ctypes.POINTER(ctypes.c_int32), _P]),
+    "cdsl_lookahead": (_I, [_P, _P, _P, _P]),
+    "cdsl_verify": (_I, [_P, _P, _P, _P, _P]),
+    "cdsl_select": (_I, [_P, _P, _P, _P, _P, _P]),
+    "cdsl_step": (_I, [_P, _P, _P, _P, _P, _P]),
+    "cdsl_get_tokens": (_I, [_P, _P, _P]),
+    "cdsl_get_counters": (_I, [_P, ctypes.POINTER(ctypes.c_int64)]),
+    "cdsl_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_int32)]),
+    "cdsl_profile": (_I, [_P, _I]),
+    "cdsl_get_profile": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double)]),
+    "cdsl_last_error": (ctypes.c_char_p, [_P]),
+    "cdsl_destroy": (None, [_P]),
+}
+
+
+def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
+    if not os.path.exists(path):
+        raise ImportError(
+            f"CUDA library {path} is missing: build it with "
+            "`python -m paper_2412_10418_gb300.build` (there is no CPU fallback)")
+    lib = ctypes.CDLL(path)
+    for name, (res, args) in EXPORTS.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib: Optional[ctypes.CDLL] = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        _lib = load_library()
+    return _lib
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _check(code: int, ctx=None):
+    if code != 0:
+        msg = lib().cdsl_last_error(ctx)
+        raise CdslError(code, msg.decode() if msg else "")
+
+
+def model_cfg(shape, dtype) -> ModelCfg:
+    """ctypes config from any object with the decoder's shape attributes."""
+    dt = dtype if isinstance(dtype, int) else (DTYPE_BF16 if dtype == "bf16" else DTYPE_F32)
+    return ModelCfg(shape.n_layers, shape.d_model, shape.n_heads, shape.n_kv_heads,
+                    shape.head_dim, shape.d_ffn, shape.vocab, dt, shape.rope_theta,
+                    shape.norm_eps)
+
+
+def run_cfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, reward_head,
+            page_size=0, max_chunk=0) -> RunCfg:
+    return RunCfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, int(reward_head),
+                  page_size, max_chunk, 0)
+
+
+# ------------------------------------------------------------------------------ C names
+
+def cdsl_num_weights(cfg: ModelCfg) -> int:
+    return lib().cdsl_num_weights(ctypes.byref(cfg))
+
+
+def cdsl_workspace_size(tcfg: ModelCfg, dcfg: ModelCfg, run: RunCfg) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().cdsl_workspace_size(ctypes.byref(tcfg), ctypes.byref(dcfg), ctypes.byref(run),
+                                     ctypes.byref(n)))
+    return n.value
+
+
+def cdsl_init(tcfg, t_weights: Sequence, dcfg, d_weights: Sequence, run, reward_head,
+              workspace, stream) -> int:
+    tw = (_P * len(t_weights))(*[w.data_ptr() for w in t_weights])
+    dw = (_P * len(d_weights))(*[w.data_ptr() for w in d_weights])
+    ctx = _P(0)
+    _check(lib().cdsl_init(ctypes.byref(tcfg), tw, ctypes.byref(dcfg), dw, ctypes.byref(run),
+                           _ptr(reward_head), workspace.data_ptr(), workspace.numel(),
+                           stream, ctypes.byref(ctx)))
+    return ctx.value
+
+
+def cdsl_prefill(ctx, prompts, prompt_lens: Sequence[int], keywords):
+    lens = (ctypes.c_int32 * len(prompt_lens))(*[int(x) for x in prompt_lens])
+    _check(lib().cdsl_prefill(ctx, prompts.data_ptr(), lens, keywords.data_ptr()), ctx)
+
+
+def cdsl_lookahead(ctx, roots=None, draft_tok=None, logq=None):
+    _check(lib().cdsl_lookahead(ctx, _ptr(roots), _ptr(draft_tok), _ptr(logq)), ctx)
+
+
+def cdsl_verify(ctx, logp=None, argmax=None, n_accept=None, logits=None):
+    _check(lib().cdsl_verify(ctx, _ptr(logp), _ptr(argmax), _ptr(n_accept), _ptr(logits)), ctx)
+
+
+def cdsl_select(ctx, beam=None, state=None, emitted=None, n_emitted=None, reward=None):
+    _check(lib().cdsl_select(ctx, _ptr(beam), _ptr(state), _ptr(emitted), _ptr(n_emitted),
+                             _ptr(reward)), ctx)
+
+
+def cdsl_step(ctx, beam=None, state=None, emitted=None, n_emitted=None, reward=None):
+    _check(lib().cdsl_step(ctx, _ptr(beam), _ptr(state), _ptr(emitted), _ptr(n_emitted),
+                           _ptr(reward)), ctx)
+
+
+def cdsl_get_tokens(ctx, tokens=None, lengths=None):
+    _check(lib().cdsl_get_tokens(ctx, _ptr(tokens), _ptr(lengths)), ctx)
+
+
+def cdsl_get_counters(ctx) -> List[int]:
+    out = (ctypes.c_int64 * 8)()
+    _check(lib().cdsl_get_counters(ctx, out), ctx)
+    return list(out)
+
+
+def cdsl_get_status(ctx) -> int:
+    v = ctypes.c_int32(0)
+    _check(lib().cdsl_get_status(ctx, ctypes.byref(v)), ctx)
+    return v.value
+
+
+def cdsl_profile(ctx, enable: bool):
+    _check(lib().cdsl_profile(ctx, int(bool(enable))), ctx)
+
+
+GEMM_IMPLS = {0: "gemm_simt", 1: "gemv_stream", 2: "gemm_tc"}
+
+
+def cdsl_get_profile(ctx, impl: int):
+    out = (ctypes.c_double * 4)()
+    _check(lib().cdsl_get_profile(ctx, impl, out), ctx)
+    return dict(launches=int(out[0]), ms=out[1], bytes=out[2], flops=out[3])
+
+
+def cdsl_last_error(ctx=None) -> str:
+    m = lib().cdsl_last_error(ctx)
+    return m.decode() if m else ""
+
+
+def cdsl_destroy(ctx):
+    lib().cdsl_destroy(ctx)
+
+
+# ------------------------------------------------------------------------------ Engine
+
+class Engine:
+    """A context plus its workspace and per-step output tensors (all on one CUDA device).
+
+    target_weights / draft_weights: torch tensors in the C ABI order (cdsl_num_weights of
+    them), kept referenced for the engine's lifetime."""
+
+    def __init__(self, target_shape, draft_shape, dtype, target_weights, draft_weights, *,
+                 batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, reward_head=None,
+                 page_size=0, max_chunk=0, stream=None, device="cuda"):
+        import torch
+
+        self.torch = torch
+        self.tcfg = model_cfg(target_shape, dtype)
+        self.dcfg = model_cfg(draft_shape, dtype)
+        self.run = run_cfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t,
+                           reward_head is not None, page_size, max_chunk)
+        self.B, self.k, self.d, self.V = batch, k, d, target_shape.vocab
+        self.max_prompt, self.max_new = max_prompt, max_new
+        self.tw, self.dw = list(target_weights), list(draft_weights)
+        self.head = reward_head
+        self.stream = stream if stream is not None else torch.cuda.Stream(device=device)
+        nbytes = cdsl_workspace_size(self.tcfg, self.dcfg, self.run)
+        self.ws = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        self.ctx = cdsl_init(self.tcfg, self.tw, self.dcfg, self.dw, self.run, self.head, self.ws,
+                             self.stream.cuda_stream)
+        i32, f32 = torch.int32, torch.float32
+        B, K, D = batch, k, d
+        z = lambda *s, dt=i32: torch.zeros(s, dtype=dt, device=device)
+        self.roots, self.draft_tok, self.logq = z(B, K), z(B, K, D), z(B, K, D, dt=f32)
+        self.logp, self.argmax, self.n_accept = z(B, K, D, dt=f32), z(B, K, D + 1), z(B, K)
+        self.beam, self.state, self.emitted = z(B), z(B), z(B, D + 1)
+        self.n_emitted, self.reward = z(B), z(B, K, 2, dt=f32)
+
+    def prefill(self, prompts, prompt_lens, keywords):
+        with self.torch.cuda.stream(self.stream):
+            self._prompts = prompts.to(self.ws.device, self.torch.int32).contiguous()
+            self._kw = keywords.to(self.ws.device, self.torch.int32).contiguous()
+        self.stream.synchronize()
+        cdsl_prefill(self.ctx, self._prompts, prompt_lens, self._kw)
+
+    def lookahead(self):
+        cdsl_lookahead(self.ctx, self.roots, self.draft_tok, self.logq)
+
+    def verify(self, logits=None):
+        cdsl_verify(self.ctx, self.logp, self.argmax, self.n_accept, logits)
+
+    def select(self):
+        cdsl_select(self.ctx, self.beam, self.state, self.emitted, self.n_emitted, self.reward)
+
+    def step(self):
+        cdsl_step(self.ctx, self.beam, self.state, self.emitted, self.n_emitted, self.reward)
+
+    def tokens(self):
+        t = self.torch.empty((self.B, self.max_prompt + self.max_new), dtype=self.torch.int32,
+                             device=self.ws.device)
+        n = self.torch.empty(self.B, dtype=self.torch.int32, device=self.ws.device)
+        cdsl_get_tokens(self.ctx, t, n)
+        self.stream.synchronize()
+        return t, n
+
+    def counters(self):
+        return cdsl_get_counters(self.ctx)
+
+    def status(self):
+        return cdsl_get_status(self.ctx)
+
+    def close(self):
+        if getattr(self, "ctx", None):
+            cdsl_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

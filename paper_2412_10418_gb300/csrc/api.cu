@@ -1,0 +1,711 @@
+// api.cu -- the C ABI of include/cdsl.h: context, workspace layout, forward passes of the
+// draft and target models, and the CDSL-k step (lookahead, verify, select) on one stream.
+#include <cuda_runtime.h>
+
+#include <array>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "kernels.h"
+
+using namespace cdsl;
+
+namespace {
+
+thread_local std::string g_init_error;
+
+enum Phase { PH_NEW = 0, PH_READY = 1, PH_LOOKED = 2, PH_VERIFIED = 3 };
+
+struct ModelW {
+  cdsl_model_cfg cfg{};
+  const void* embed = nullptr;
+  const void* final_norm = nullptr;
+  const void* lm_head = nullptr;
+  std::vector<std::array<const void*, 9>> layers;
+  KvStore kv{};
+  float2* rope = nullptr;
+  int32_t spb = 0;  // tail slots per beam
+};
+
+enum { W_ATTN_NORM = 0, W_Q, W_K, W_V, W_O, W_FFN_NORM, W_GATE, W_UP, W_DOWN };
+
+// Bump allocator over the caller's workspace; with base == nullptr it only measures.
+struct Carver {
+  char* base;
+  size_t off = 0;
+  explicit Carver(void* b) : base(static_cast<char*>(b)) {}
+  template <typename T>
+  T* take(size_t count) {
+    off = (off + 255) & ~size_t(255);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+}  // namespace
+
+struct cdsl_ctx {
+  cdsl_model_cfg tcfg{}, dcfg{};
+  cdsl_run_cfg run{};
+  ModelW tgt, dft;
+  cudaStream_t stream = nullptr;
+  const float* head_w = nullptr;
+  int dtype = 0;
+  int B = 0, k = 0, d = 0, nk = 0, lcap = 0, lrope = 0, max_pages = 0, page_shift = 0;
+  int R_v = 0, R_d = 0, R_p = 0, R_max = 0, R_pad = 0, V = 0;
+  int d_max = 0, act_cols = 0, q_cols = 0;
+  size_t act_plane = 0;  // elements between hi and lo planes of X1 / X2 (bf16 models)
+  // buffers
+  float* h = nullptr;
+  void* X1 = nullptr;
+  void* X2 = nullptr;
+  float* qbuf = nullptr;
+  float* logits = nullptr;
+  RowDesc* rows_d = nullptr;
+  RowDesc* rows_v = nullptr;
+  RowDesc* rows_p = nullptr;
+  int32_t* lm_gather = nullptr;
+  int32_t* lm_dst = nullptr;
+  StepState st{};
+  size_t ws_total = 0;
+  int phase = PH_NEW;
+  cudaGraphExec_t graph = nullptr;
+  long long graph_nodes = 0;
+  // kernel timing (cdsl_profile)
+  struct ProfRec { int impl; double bytes, flops; size_t ev; };
+  bool profiling = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  std::vector<ProfRec> prof;
+  std::string err;
+};
+
+namespace {
+
+int fail(cdsl_ctx* c, int code, const std::string& msg) {
+  if (c) c->err = msg; else g_init_error = msg;
+  return code;
+}
+
+int cuda_check(cdsl_ctx* c, const char* where) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess)
+    return fail(c, CDSL_ECUDA, std::string(where) + ": " + cudaGetErrorString(e));
+  return CDSL_OK;
+}
+
+int check_model(const cdsl_model_cfg* m, const char* name, std::string* why) {
+  char buf[256];
+  auto bad = [&](const char* what) {
+    snprintf(buf, sizeof buf, "%s config: %s", name, what);
+    *why = buf;
+    return CDSL_EINVAL;
+  };
+  if (!m) return bad("NULL");
+  if (m->n_layers < 1 || m->n_layers > 512) return bad("n_layers out of range");
+  if (m->d_model < 64 || m->d_model % 64) return bad("d_model must be a positive multiple of 64");
+  if (m->head_dim != 64 && m->head_dim != 128) return bad("head_dim must be 64 or 128");
+  if (m->n_heads < 1 || m->n_kv_heads < 1 || m->n_heads % m->n_kv_heads)
+    return bad("n_heads must be a positive multiple of n_kv_heads");
+  if (m->n_heads / m->n_kv_heads > 16) return bad("more than 16 query heads per kv head");
+  if (m->d_ffn < 8 || m->d_ffn % 8) return bad("d_ffn must be a positive multiple of 8");
+  if (m->vocab < 2 || m->vocab % 8) return bad("vocab must be a multiple of 8");
+  if (m->dtype != CDSL_DTYPE_F32 && m->dtype != CDSL_DTYPE_BF16) return bad("unknown dtype");
+  if (!(m->rope_theta > 0.f) || !(m->norm_eps > 0.f)) return bad("rope_theta and norm_eps must be > 0");
+  return CDSL_OK;
+}
+
+int check_run(const cdsl_run_cfg* r, int vocab, std::string* why) {
+  auto bad = [&](const char* what) { *why = std::string("run config: ") + what; return CDSL_EINVAL; };
+  if (!r) return bad("NULL");
+  if (r->batch < 1 || r->batch > 4096) return bad("batch out of range");
+  if (r->k < 1 || r->k > 16 || r->k > vocab) return bad("k must be in 1..16");
+  if (r->d < 1 || r->d > 16) return bad("d must be in 1..16");
+  if (r->max_prompt < 1 || r->max_new < 1) return bad("max_prompt and max_new must be >= 1");
+  if ((long long)r->max_prompt + r->max_new > (1 << 20)) return bad("sequence too long");
+  if (r->n_keywords < 1 || r->n_keywords > 32) return bad("n_keywords must be in 1..32");
+  const int ps = r->page_size ? r->page_size : 64;
+  if (ps < 16 || ps > 256 || (ps & (ps - 1))) return bad("page_size must be a power of two in 16..256");
+  if (r->max_chunk < 0) return bad("max_chunk must be >= 0");
+  return CDSL_OK;
+}
+
+// Sizes derived from the configurations (shared by cdsl_workspace_size and cdsl_init).
+void derive_dims(cdsl_ctx* c) {
+  const cdsl_run_cfg& r = c->run;
+  c->dtype = c->tcfg.dtype;
+  c->B = r.batch; c->k = r.k; c->d = r.d; c->nk = r.n_keywords;
+  c->V = c->tcfg.vocab;
+  c->lcap = r.max_prompt + r.max_new + 1;
+  c->lrope = r.max_prompt + r.max_new + r.d + 2;
+  const int ps = r.page_size ? r.page_size : 64;
+  c->page_shift = 0;
+  while ((1 << c->page_shift) < ps) ++c->page_shift;
+  c->max_pages = (c->lcap + ps - 1) / ps;
+  c->R_v = c->B * c->k * (c->d + 1);
+  c->R_d = c->B * c->k + c->B;
+  const int chunk = r.max_chunk ? r.max_chunk : 256;
+  c->R_p = std::min(chunk, c->B * r.max_prompt);
+  c->R_max = std::max(c->R_v, std::max(c->R_d, c->R_p));
+  c->R_pad = (c->R_max + 31) / 32 * 32;
+  c->d_max = std::max(c->tcfg.d_model, c->dcfg.d_model);
+  c->q_cols = std::max(c->tcfg.n_heads * c->tcfg.head_dim, c->dcfg.n_heads * c->dcfg.head_dim);
+  c->act_cols = std::max(std::max(c->d_max, c->q_cols), std::max(c->tcfg.d_ffn, c->dcfg.d_ffn));
+}
+
+KvStore make_kv(const cdsl_model_cfg& m, cdsl_ctx* c, int slots) {
+  KvStore s{};
+  s.n_pages = c->B * c->max_pages;
+  s.page_shift = c->page_shift;
+  s.max_pages = c->max_pages;
+  s.kvh = m.n_kv_heads;
+  s.hd = m.head_dim;
+  s.n_tail_slots = slots;
+  s.n_layers = m.n_layers;
+  return s;
+}
+
+// Carve every buffer; returns total bytes. With base == nullptr only the size is computed.
+size_t carve(cdsl_ctx* c, void* base) {
+  Carver cv(base);
+  const int B = c->B, k = c->k, d = c->d;
+  auto model_kv = [&](ModelW& m, const cdsl_model_cfg& cfg, int slots) {
+    m.kv = make_kv(cfg, c, slots);
+    const size_t per_page = (size_t)2 * cfg.n_kv_heads * ((size_t)1 << c->page_shift) * cfg.head_dim;
+    m.kv.pool = cv.take<float>((size_t)cfg.n_layers * m.kv.n_pages * per_page);
+    m.kv.tail = cv.take<float>((size_t)cfg.n_layers * 2 * slots * cfg.n_kv_heads * cfg.head_dim);
+    m.kv.page_table = cv.take<int32_t>((size_t)B * c->max_pages);
+    m.rope = cv.take<float2>((size_t)c->lrope * (cfg.head_dim / 2));
+    m.spb = slots / (B * k);
+  };
+  model_kv(c->tgt, c->tcfg, B * k * (d + 1));
+  model_kv(c->dft, c->dcfg, B * k * d);
+  c->h = cv.take<float>((size_t)c->R_pad * c->d_max);
+  // GEMM inputs: one fp32 plane, or hi/lo bf16 planes (4 bytes per element either way)
+  c->act_plane = (size_t)c->R_pad * c->act_cols;
+  c->X1 = cv.take<float>(c->act_plane);
+  c->X2 = cv.take<float>(c->act_plane);
+  c->qbuf = cv.take<float>((size_t)c->R_pad * c->q_cols);
+  const int lm_rows = std::max(c->R_v, std::max(B * k, B));
+  c->logits = cv.take<float>((size_t)lm_rows * c->V);
+  c->rows_d = cv.take<RowDesc>(c->R_d);
+  c->rows_v = cv.take<RowDesc>(c->R_v);
+  c->rows_p = cv.take<RowDesc>(c->R_p);
+  c->lm_gather = cv.take<int32_t>(c->R_p);
+  c->lm_dst = cv.take<int32_t>(c->R_p);
+  StepState& s = c->st;
+  s.B = B; s.k = k; s.d = d; s.nk = c->nk; s.max_new = c->run.max_new; s.lcap = c->lcap;
+  s.reward_head = c->run.reward_head;
+  s.r_t = c->run.r_t;
+  s.n_min = d + 1;
+  for (int n = 0; n <= d; ++n)
+    if ((float)n / (float)d >= c->run.a_t) { s.n_min = n; break; }
+  s.len = cv.take<int32_t>(B);
+  s.pend = cv.take<int32_t>(B);
+  s.gen = cv.take<int32_t>(B);
+  s.tokens = cv.take<int32_t>((size_t)B * c->lcap);
+  s.roots = cv.take<int32_t>((size_t)B * k);
+  s.kw = cv.take<int32_t>((size_t)B * c->nk);
+  s.cov = cv.take<uint32_t>(B);
+  s.x = cv.take<int32_t>((size_t)B * k * d);
+  s.logq = cv.take<float>((size_t)B * k * d);
+  s.v_amax = cv.take<int32_t>(c->R_v);
+  s.v_logp = cv.take<float>((size_t)B * k * d);
+  s.v_topk = cv.take<int32_t>((size_t)c->R_v * k);
+  s.v_head = cv.take<float>(c->R_v);
+  s.n_acc = cv.take<int32_t>((size_t)B * k);
+  s.reward = cv.take<float>((size_t)B * k * 2);
+  s.beam = cv.take<int32_t>(B);
+  s.state = cv.take<int32_t>(B);
+  s.emitted = cv.take<int32_t>((size_t)B * (d + 1));
+  s.n_emit = cv.take<int32_t>(B);
+  s.next_page = cv.take<int32_t>(2);
+  s.status = cv.take<int32_t>(1);
+  s.counters = cv.take<long long>(8);
+  return (cv.off + 255) & ~size_t(255);
+}
+
+// Algorithmic bytes of one projection GEMM: every weight once, the activations read once
+// (4 bytes per element: fp32, or bf16 hi + lo), the outputs written once (read-modify-write
+// for the residual add).
+double gemm_bytes(const cdsl_ctx* c, const GemmArgs& a, double* flops) {
+  const double wsz = c->dtype == CDSL_DTYPE_BF16 ? 2.0 : 4.0;
+  double rows = 0;
+  for (int s = 0; s < a.n_seg; ++s) rows += a.seg_rows[s];
+  *flops = 2.0 * a.R * rows * a.K;
+  double out = 0;
+  switch (a.mode) {
+    case EPI_STORE: out = 4.0 * a.R * rows; break;
+    case EPI_RESID: out = 8.0 * a.R * rows; break;
+    case EPI_SWIGLU: out = 4.0 * a.R * a.d_ffn; break;
+    case EPI_QKV: out = 4.0 * a.R * rows; break;
+  }
+  return rows * a.K * wsz + 4.0 * a.R * a.K + out;
+}
+
+void gemm(cdsl_ctx* c, const GemmArgs& a) {
+  const int impl = 0;
+  size_t ev = 0;
+  if (c->profiling) {
+    while (c->ev_pool.size() < c->ev_used + 2) {
+      cudaEvent_t e;
+      cudaEventCreate(&e);
+      c->ev_pool.push_back(e);
+    }
+    ev = c->ev_used;
+    c->ev_used += 2;
+    cudaEventRecord(c->ev_pool[ev], c->stream);
+  }
+  launch_gemm_simt(c->dtype, a, c->stream);
+  if (c->profiling) {
+    cudaEventRecord(c->ev_pool[ev + 1], c->stream);
+    double fl = 0;
+    const double by = gemm_bytes(c, a, &fl);
+    c->prof.push_back({impl, by, fl, ev});
+  }
+}
+
+GemmArgs gemm_base(const cdsl_ctx* c, const ModelW& m, int mode, int K, const void* x, int ldx,
+                   int R) {
+  GemmArgs a{};
+  a.mode = mode;
+  a.K = K;
+  a.x = x;
+  a.ldx = ldx;
+  a.x_plane = (int64_t)c->act_plane;
+  a.act_plane = (int64_t)c->act_plane;
+  a.R = R;
+  a.n_heads = m.cfg.n_heads;
+  a.kv = m.kv;
+  return a;
+}
+
+// One forward pass of a model over R rows described by `rows`; for lm_rows > 0 the final
+// norm + LM head run over rows gather[i] (or the first lm_rows rows) into logits.
+void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
+             const int32_t* gather, float* logits, float* head_out) {
+  const cdsl_model_cfg& cfg = m.cfg;
+  const int D = cfg.d_model, hd = cfg.head_dim, H = cfg.n_heads, KVH = cfg.n_kv_heads;
+  const int F = cfg.d_ffn;
+  cudaStream_t s = c->stream;
+  launch_embed(c->dtype, rows, R, m.embed, D, c->h, s);
+  for (int l = 0; l < cfg.n_layers; ++l) {
+    const auto& W = m.layers[l];
+    launch_rmsnorm(c->dtype, c->h, R, D, W[W_ATTN_NORM], cfg.norm_eps, c->X1, c->act_plane,
+                   nullptr, nullptr, nullptr, s);
+    GemmArgs q = gemm_base(c, m, EPI_QKV, D, c->X1, D, R);
+    q.w[0] = W[W_Q]; q.w[1] = W[W_K]; q.w[2] = W[W_V];
+    q.seg_rows[0] = H * hd; q.seg_rows[1] = KVH * hd; q.seg_rows[2] = KVH * hd;
+    q.n_seg = 3;
+    q.n_virtual = (H + 2 * KVH) * hd;
+    q.q_out = c->qbuf;
+    q.layer = l;
+    q.rows = rows;
+    q.rope = m.rope;
+    gemm(c, q);
+    launch_attention(c->dtype, c->qbuf, m.kv, l, rows, R, H, c->lcap + c->d + 1, c->X1,
+                     c->act_plane, c->st.status, s);
+    GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->X1, H * hd, R);
+    o.w[0] = W[W_O]; o.seg_rows[0] = D; o.n_seg = 1; o.n_virtual = D;
+    o.out_f32 = c->h; o.ld_out = D;
+    gemm(c, o);
+    launch_rmsnorm(c->dtype, c->h, R, D, W[W_FFN_NORM], cfg.norm_eps, c->X1, c->act_plane,
+                   nullptr, nullptr, nullptr, s);
+    GemmArgs g = gemm_base(c, m, EPI_SWIGLU, D, c->X1, D, R);
+    g.w[0] = W[W_GATE]; g.w[1] = W[W_UP]; g.seg_rows[0] = F; g.seg_rows[1] = F; g.n_seg = 2;
+    g.n_virtual = (F + 63) / 64 * 128;
+    g.d_ffn = F;
+    g.out_act = c->X2; g.ld_act = F;
+    gemm(c, g);
+    GemmArgs dn = gemm_base(c, m, EPI_RESID, F, c->X2, F, R);
+    dn.w[0] = W[W_DOWN]; dn.seg_rows[0] = D; dn.n_seg = 1; dn.n_virtual = D;
+    dn.out_f32 = c->h; dn.ld_out = D;
+    gemm(c, dn);
+  }
+  if (lm_rows > 0) {
+    launch_rmsnorm(c->dtype, c->h, lm_rows, D, m.final_norm, cfg.norm_eps, c->X1, c->act_plane,
+                   gather, head_out ? c->head_w : nullptr, head_out, s);
+    GemmArgs lm = gemm_base(c, m, EPI_STORE, D, c->X1, D, lm_rows);
+    lm.w[0] = m.lm_head; lm.seg_rows[0] = cfg.vocab; lm.n_seg = 1; lm.n_virtual = cfg.vocab;
+    lm.out_f32 = logits; lm.ld_out = cfg.vocab;
+    gemm(c, lm);
+  }
+}
+
+void do_lookahead(cdsl_ctx* c) {
+  for (int j = 1; j <= c->d; ++j) {
+    launch_plan_draft(c->st, j, c->dft.spb, c->rows_d, c->stream);
+    const int R = c->B * c->k + (j == 1 ? c->B : 0);
+    forward(c, c->dft, c->rows_d, R, c->B * c->k, nullptr, c->logits, nullptr);
+    RowStatsArgs a{};
+    a.logits = c->logits; a.R = c->B * c->k; a.V = c->V; a.k = c->k;
+    a.x_out = c->st.x; a.logq_out = c->st.logq; a.out_stride = c->d; a.out_off = j - 1;
+    a.status = c->st.status;
+    launch_row_stats(a, c->stream);
+  }
+}
+
+void do_verify(cdsl_ctx* c) {
+  launch_plan_verify(c->st, c->rows_v, c->stream);
+  forward(c, c->tgt, c->rows_v, c->R_v, c->R_v, nullptr, c->logits,
+          c->run.reward_head ? c->st.v_head : nullptr);
+  RowStatsArgs a{};
+  a.logits = c->logits; a.R = c->R_v; a.V = c->V; a.k = c->k; a.dp1 = c->d + 1;
+  a.next_x = c->st.x; a.amax = c->st.v_amax; a.logp = c->st.v_logp; a.topk = c->st.v_topk;
+  a.status = c->st.status;
+  launch_row_stats(a, c->stream);
+}
+
+void do_select(cdsl_ctx* c) {
+  launch_select(c->st, c->tgt.kv, c->dft.kv, 1, c->stream);
+  launch_commit_kv(c->st, c->tgt.kv, c->tgt.spb, 0, c->stream);
+  launch_commit_kv(c->st, c->dft.kv, c->dft.spb, 1, c->stream);
+  launch_advance(c->st, c->stream);
+}
+
+void copy_out(cdsl_ctx* c, void* dst, const void* src, size_t bytes) {
+  if (dst) cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, c->stream);
+}
+
+void copy_select_outputs(cdsl_ctx* c, int32_t* beam, int32_t* state, int32_t* emitted,
+                         int32_t* n_emitted, float* reward) {
+  const size_t B = c->B;
+  copy_out(c, beam, c->st.beam, B * 4);
+  copy_out(c, state, c->st.state, B * 4);
+  copy_out(c, emitted, c->st.emitted, B * (c->d + 1) * 4);
+  copy_out(c, n_emitted, c->st.n_emit, B * 4);
+  copy_out(c, reward, c->st.reward, B * c->k * 2 * 4);
+}
+
+int bind_model(ModelW& m, const cdsl_model_cfg& cfg, const void* const* w, const char* name,
+               std::string* why) {
+  const int n = cdsl_num_weights(&cfg);
+  for (int i = 0; i < n; ++i) {
+    if (!w[i] || (reinterpret_cast<uintptr_t>(w[i]) & 15)) {
+      char buf[160];
+      snprintf(buf, sizeof buf, "%s weight %d is NULL or not 16-byte aligned", name, i);
+      *why = buf;
+      return CDSL_EINVAL;
+    }
+  }
+  m.cfg = cfg;
+  m.embed = w[0];
+  m.layers.resize(cfg.n_layers);
+  for (int l = 0; l < cfg.n_layers; ++l)
+    for (int j = 0; j < 9; ++j) m.layers[l][j] = w[1 + 9 * l + j];
+  m.final_norm = w[1 + 9 * cfg.n_layers];
+  m.lm_head = w[2 + 9 * cfg.n_layers];
+  return CDSL_OK;
+}
+
+int validate_all(const cdsl_model_cfg* t, const cdsl_model_cfg* dr, const cdsl_run_cfg* r,
+                 std::string* why) {
+  int e = check_model(t, "target", why);
+  if (e) return e;
+  if ((e = check_model(dr, "draft", why))) return e;
+  if (t->vocab != dr->vocab) { *why = "target and draft vocabularies differ"; return CDSL_EINVAL; }
+  if (t->dtype != dr->dtype) { *why = "target and draft dtypes differ"; return CDSL_EINVAL; }
+  return check_run(r, t->vocab, why);
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t cdsl_num_weights(const cdsl_model_cfg* cfg) {
+  if (!cfg || cfg->n_layers < 1) return -1;
+  return 3 + 9 * cfg->n_layers;
+}
+
+int32_t cdsl_workspace_size(const cdsl_model_cfg* target, const cdsl_model_cfg* draft,
+                            const cdsl_run_cfg* run, size_t* bytes) {
+  std::string why;
+  int e = validate_all(target, draft, run, &why);
+  if (e) return fail(nullptr, e, why);
+  if (!bytes) return fail(nullptr, CDSL_EINVAL, "bytes is NULL");
+  cdsl_ctx tmp;
+  tmp.tcfg = *target; tmp.dcfg = *draft; tmp.run = *run;
+  derive_dims(&tmp);
+  *bytes = carve(&tmp, nullptr);
+  return CDSL_OK;
+}
+
+int32_t cdsl_init(const cdsl_model_cfg* target, const void* const* h_target_weights,
+                  const cdsl_model_cfg* draft, const void* const* h_draft_weights,
+                  const cdsl_run_cfg* run, const float* d_reward_head, void* d_workspace,
+                  size_t workspace_bytes, void* stream, cdsl_ctx** out) {
+  std::string why;
+  int e = validate_all(target, draft, run, &why);
+  if (e) return fail(nullptr, e, why);
+  if (!out) return fail(nullptr, CDSL_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (!h_target_weights || !h_draft_weights) return fail(nullptr, CDSL_EINVAL, "weights are NULL");
+  if (run->reward_head && !d_reward_head)
+    return fail(nullptr, CDSL_EINVAL, "reward_head requested but d_reward_head is NULL");
+  if (!d_workspace || (reinterpret_cast<uintptr_t>(d_workspace) & 255))
+    return fail(nullptr, CDSL_EINVAL, "workspace is NULL or not 256-byte aligned");
+  cdsl_ctx* c = new cdsl_ctx();
+  c->tcfg = *target; c->dcfg = *draft; c->run = *run;
+  c->head_w = d_reward_head;
+  c->stream = static_cast<cudaStream_t>(stream);
+  derive_dims(c);
+  if ((e = bind_model(c->tgt, *target, h_target_weights, "target", &why)) ||
+      (e = bind_model(c->dft, *draft, h_draft_weights, "draft", &why))) {
+    delete c;
+    return fail(nullptr, e, why);
+  }
+  c->ws_total = carve(c, nullptr);
+  if (workspace_bytes < c->ws_total) {
+    char buf[160];
+    snprintf(buf, sizeof buf, "workspace has %zu bytes, needs %zu", workspace_bytes, c->ws_total);
+    delete c;
+    return fail(nullptr, CDSL_ENOMEM, buf);
+  }
+  carve(c, d_workspace);
+  cudaGetLastError();
+  cudaMemsetAsync(d_workspace, 0, c->ws_total, c->stream);
+  launch_rope_table(c->tgt.rope, c->lrope, target->head_dim, target->rope_theta, c->stream);
+  launch_rope_table(c->dft.rope, c->lrope, draft->head_dim, draft->rope_theta, c->stream);
+  if ((e = cuda_check(c, "cdsl_init"))) {
+    g_init_error = c->err;
+    delete c;
+    return e;
+  }
+  c->phase = PH_NEW;
+  *out = c;
+  return CDSL_OK;
+}
+
+int32_t cdsl_prefill(cdsl_ctx* c, const int32_t* d_prompts, const int32_t* h_prompt_lens,
+                     const int32_t* d_keywords) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (!d_prompts || !h_prompt_lens || !d_keywords)
+    return fail(c, CDSL_EINVAL, "prompts, prompt lengths and keywords are required");
+  const int B = c->B, P = 1 << c->page_shift;
+  for (int b = 0; b < B; ++b)
+    if (h_prompt_lens[b] < 1 || h_prompt_lens[b] > c->run.max_prompt)
+      return fail(c, CDSL_EINVAL, "prompt length out of 1..max_prompt");
+  cudaStream_t s = c->stream;
+  StepState& st = c->st;
+  cudaGetLastError();
+  // reset the decoding state
+  cudaMemsetAsync(st.tokens, 0xff, sizeof(int32_t) * B * c->lcap, s);
+  cudaMemsetAsync(st.pend, 0, sizeof(int32_t) * B, s);
+  cudaMemsetAsync(st.gen, 0, sizeof(int32_t) * B, s);
+  cudaMemsetAsync(st.cov, 0, sizeof(uint32_t) * B, s);
+  cudaMemsetAsync(st.status, 0, sizeof(int32_t), s);
+  cudaMemsetAsync(st.counters, 0, sizeof(long long) * 8, s);
+  cudaMemcpy2DAsync(st.tokens, sizeof(int32_t) * c->lcap, d_prompts,
+                    sizeof(int32_t) * c->run.max_prompt, sizeof(int32_t) * c->run.max_prompt, B,
+                    cudaMemcpyDeviceToDevice, s);
+  cudaMemcpyAsync(st.len, h_prompt_lens, sizeof(int32_t) * B, cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(st.kw, d_keywords, sizeof(int32_t) * B * c->nk, cudaMemcpyDeviceToDevice, s);
+  // pages for the prompts: contiguous runs handed out in prompt order
+  std::vector<int32_t> pt((size_t)B * c->max_pages, -1);
+  int next = 0;
+  for (int b = 0; b < B; ++b)
+    for (int p = 0; p < (h_prompt_lens[b] + P - 1) / P; ++p) pt[(size_t)b * c->max_pages + p] = next++;
+  int32_t np[2] = {next, next};
+  cudaMemcpyAsync(c->tgt.kv.page_table, pt.data(), pt.size() * 4, cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(c->dft.kv.page_table, pt.data(), pt.size() * 4, cudaMemcpyHostToDevice, s);
+  cudaMemcpyAsync(st.next_page, np, sizeof np, cudaMemcpyHostToDevice, s);
+  // causal prompt rows, in chunks of at most R_p rows
+  std::vector<RowDesc> rows;
+  std::vector<int32_t> gather, dst;
+  auto flush = [&]() {
+    if (rows.empty()) return;
+    const int R = (int)rows.size();
+    cudaMemcpyAsync(c->rows_p, rows.data(), sizeof(RowDesc) * R, cudaMemcpyHostToDevice, s);
+    const int nlm = (int)gather.size();
+    if (nlm) {
+      cudaMemcpyAsync(c->lm_gather, gather.data(), 4 * nlm, cudaMemcpyHostToDevice, s);
+      cudaMemcpyAsync(c->lm_dst, dst.data(), 4 * nlm, cudaMemcpyHostToDevice, s);
+    }
+    forward(c, c->tgt, c->rows_p, R, nlm, c->lm_gather, c->logits, nullptr);
+    if (nlm) {
+      RowStatsArgs a{};
+      a.logits = c->logits; a.R = nlm; a.V = c->V; a.k = c->k;
+      a.topk = st.roots; a.dst = c->lm_dst; a.status = st.status;
+      launch_row_stats(a, s);
+    }
+    forward(c, c->dft, c->rows_p, R, 0, nullptr, nullptr, nullptr);
+    cudaStreamSynchronize(s);  // host row buffers are reused by the next chunk
+    rows.clear(); gather.clear(); dst.clear();
+  };
+  std::vector<int32_t> host_tokens((size_t)B * c->run.max_prompt);
+  cudaMemcpyAsync(host_tokens.data(), d_prompts, host_tokens.size() * 4, cudaMemcpyDeviceToHost, s);
+  cudaStreamSynchronize(s);
+  for (int b = 0; b < B; ++b) {
+    for (int p = 0; p < h_prompt_lens[b]; ++p) {
+      const int32_t tok = host_tokens[(size_t)b * c->run.max_prompt + p];
+      if (tok < 0 || tok >= c->V) return fail(c, CDSL_EINVAL, "prompt token id out of range");
+      RowDesc rd{};
+      rd.b = b; rd.pos = p; rd.token = tok; rd.n_prefix = p + 1; rd.tail_base = 0; rd.n_tail = 0;
+      rd.kv_dst = KV_PREFIX; rd.out_idx = (p == h_prompt_lens[b] - 1) ? b : -1;
+      if (rd.out_idx >= 0) { gather.push_back((int)rows.size()); dst.push_back(b); }
+      rows.push_back(rd);
+      if ((int)rows.size() == c->R_p) flush();
+    }
+  }
+  flush();
+  int e = cuda_check(c, "cdsl_prefill");
+  if (e) return e;
+  c->phase = PH_READY;
+  return CDSL_OK;
+}
+
+int32_t cdsl_lookahead(cdsl_ctx* c, int32_t* d_roots, int32_t* d_draft_tok, float* d_logq) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (c->phase != PH_READY) return fail(c, CDSL_ESTATE, "cdsl_lookahead needs a prefilled context");
+  cudaGetLastError();
+  do_lookahead(c);
+  const size_t n = (size_t)c->B * c->k;
+  copy_out(c, d_roots, c->st.roots, n * 4);
+  copy_out(c, d_draft_tok, c->st.x, n * c->d * 4);
+  copy_out(c, d_logq, c->st.logq, n * c->d * 4);
+  int e = cuda_check(c, "cdsl_lookahead");
+  if (e) return e;
+  c->phase = PH_LOOKED;
+  return CDSL_OK;
+}
+
+int32_t cdsl_verify(cdsl_ctx* c, float* d_logp, int32_t* d_argmax, int32_t* d_n_accept,
+                    float* d_logits) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (c->phase != PH_LOOKED) return fail(c, CDSL_ESTATE, "cdsl_verify needs a preceding cdsl_lookahead");
+  cudaGetLastError();
+  do_verify(c);
+  const size_t n = (size_t)c->B * c->k;
+  copy_out(c, d_logp, c->st.v_logp, n * c->d * 4);
+  copy_out(c, d_argmax, c->st.v_amax, n * (c->d + 1) * 4);
+  copy_out(c, d_logits, c->logits, (size_t)c->R_v * c->V * 4);
+  if (d_n_accept) {
+    // n_b is settled by the decision kernel; run it here without committing anything.
+    launch_select(c->st, c->tgt.kv, c->dft.kv, 0, c->stream);
+    copy_out(c, d_n_accept, c->st.n_acc, n * 4);
+  }
+  int e = cuda_check(c, "cdsl_verify");
+  if (e) return e;
+  c->phase = PH_VERIFIED;
+  return CDSL_OK;
+}
+
+int32_t cdsl_select(cdsl_ctx* c, int32_t* d_beam, int32_t* d_state, int32_t* d_emitted,
+                    int32_t* d_n_emitted, float* d_reward) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (c->phase != PH_VERIFIED) return fail(c, CDSL_ESTATE, "cdsl_select needs a preceding cdsl_verify");
+  cudaGetLastError();
+  do_select(c);
+  copy_select_outputs(c, d_beam, d_state, d_emitted, d_n_emitted, d_reward);
+  int e = cuda_check(c, "cdsl_select");
+  if (e) return e;
+  c->phase = PH_READY;
+  return CDSL_OK;
+}
+
+int32_t cdsl_step(cdsl_ctx* c, int32_t* d_beam, int32_t* d_state, int32_t* d_emitted,
+                  int32_t* d_n_emitted, float* d_reward) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (c->phase != PH_READY) return fail(c, CDSL_ESTATE, "cdsl_step needs a prefilled context");
+  cudaGetLastError();
+  if (c->stream == nullptr || c->profiling) {  // legacy stream / timing: launch directly
+    do_lookahead(c);
+    do_verify(c);
+    do_select(c);
+  } else {
+    if (!c->graph) {
+      cudaGraph_t g = nullptr;
+      if (cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+        return fail(c, CDSL_ECUDA, "cudaStreamBeginCapture failed");
+      do_lookahead(c);
+      do_verify(c);
+      do_select(c);
+      cudaError_t ce = cudaStreamEndCapture(c->stream, &g);
+      if (ce != cudaSuccess) return fail(c, CDSL_ECUDA, std::string("capture: ") + cudaGetErrorString(ce));
+      size_t nodes = 0;
+      cudaGraphGetNodes(g, nullptr, &nodes);
+      c->graph_nodes = (long long)nodes;
+      ce = cudaGraphInstantiate(&c->graph, g, 0);
+      cudaGraphDestroy(g);
+      if (ce != cudaSuccess) {
+        c->graph = nullptr;
+        return fail(c, CDSL_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+      }
+    }
+    cudaGraphLaunch(c->graph, c->stream);
+  }
+  copy_select_outputs(c, d_beam, d_state, d_emitted, d_n_emitted, d_reward);
+  return cuda_check(c, "cdsl_step");
+}
+
+int32_t cdsl_get_tokens(cdsl_ctx* c, int32_t* d_tokens, int32_t* d_lengths) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  const int W = c->run.max_prompt + c->run.max_new;
+  if (d_tokens)
+    cudaMemcpy2DAsync(d_tokens, sizeof(int32_t) * W, c->st.tokens, sizeof(int32_t) * c->lcap,
+                      sizeof(int32_t) * W, c->B, cudaMemcpyDeviceToDevice, c->stream);
+  copy_out(c, d_lengths, c->st.len, sizeof(int32_t) * c->B);
+  return cuda_check(c, "cdsl_get_tokens");
+}
+
+int32_t cdsl_get_counters(cdsl_ctx* c, int64_t* h_counters) {
+  if (!c || !h_counters) return fail(c, CDSL_EINVAL, "ctx or counters is NULL");
+  long long tmp[8];
+  cudaMemcpyAsync(tmp, c->st.counters, sizeof tmp, cudaMemcpyDeviceToHost, c->stream);
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return cuda_check(c, "cdsl_get_counters");
+  for (int i = 0; i < 6; ++i) h_counters[i] = tmp[i];
+  h_counters[6] = c->graph_nodes;
+  h_counters[7] = 0;
+  return CDSL_OK;
+}
+
+int32_t cdsl_profile(cdsl_ctx* c, int32_t enable) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  c->profiling = enable != 0;
+  c->ev_used = 0;
+  c->prof.clear();
+  return CDSL_OK;
+}
+
+int32_t cdsl_get_profile(cdsl_ctx* c, int32_t impl, double* h_out) {
+  if (!c || !h_out) return fail(c, CDSL_EINVAL, "ctx or out is NULL");
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return fail(c, CDSL_ECUDA, std::string("cdsl_get_profile: ") + cudaGetErrorString(e));
+  double n = 0, ms = 0, by = 0, fl = 0;
+  for (const auto& r : c->prof) {
+    if (r.impl != impl) continue;
+    float t = 0;
+    cudaEventElapsedTime(&t, c->ev_pool[r.ev], c->ev_pool[r.ev + 1]);
+    n += 1; ms += t; by += r.bytes; fl += r.flops;
+  }
+  h_out[0] = n; h_out[1] = ms; h_out[2] = by; h_out[3] = fl;
+  c->ev_used = 0;
+  c->prof.clear();
+  return cuda_check(c, "cdsl_get_profile");
+}
+
+int32_t cdsl_get_status(cdsl_ctx* c, int32_t* h_device_status) {
+  if (!c || !h_device_status) return fail(c, CDSL_EINVAL, "ctx or status is NULL");
+  int32_t v = 0;
+  cudaMemcpyAsync(&v, c->st.status, sizeof v, cudaMemcpyDeviceToHost, c->stream);
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return fail(c, CDSL_ECUDA, std::string("cdsl_get_status: ") + cudaGetErrorString(e));
+  *h_device_status = v;
+  return CDSL_OK;
+}
+
+const char* cdsl_last_error(const cdsl_ctx* c) {
+  return c ? c->err.c_str() : g_init_error.c_str();
+}
+
+void cdsl_destroy(cdsl_ctx* c) {
+  if (!c) return;
+  if (c->graph) cudaGraphExecDestroy(c->graph);
+  for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
+  delete c;
+}
+
+}  // extern "C"

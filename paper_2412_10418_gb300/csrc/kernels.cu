@@ -1,0 +1,482 @@
+// kernels.cu -- embedding, RMSNorm (+ reward head), attention over the paged prefix and the
+// beam tails, logits row statistics, row plans, and the CDSL acceptance decision / commit.
+#include <cuda_bf16.h>
+#include <math.h>
+
+#include "kernels.h"
+
+namespace cdsl {
+
+namespace {
+
+constexpr int kMaxWarps = 32;
+
+__device__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[wid] = v;
+  __syncthreads();
+  float t = (threadIdx.x < nw) ? red[threadIdx.x] : 0.f;
+  if (wid == 0) t = warp_sum(t);
+  if (threadIdx.x == 0) red[0] = t;
+  __syncthreads();
+  return red[0];
+}
+
+__device__ unsigned long long block_max_u64(unsigned long long v, unsigned long long* red) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  v = warp_max_u64(v);
+  __syncthreads();
+  if (lane == 0) red[wid] = v;
+  __syncthreads();
+  unsigned long long t = (threadIdx.x < nw) ? red[threadIdx.x] : 0ull;
+  if (wid == 0) t = warp_max_u64(t);
+  if (threadIdx.x == 0) red[0] = t;
+  __syncthreads();
+  return red[0];
+}
+
+// ------------------------------------------------------------------------------ embedding
+template <typename T>
+__global__ void k_embed(const RowDesc* rows, const T* E, int D, float* h) {
+  const int r = blockIdx.x;
+  const T* e = E + (size_t)rows[r].token * D;
+  for (int c = threadIdx.x; c < D; c += blockDim.x) h[(size_t)r * D + c] = to_f32<T>(e[c]);
+}
+
+// ------------------------------------------------------------------------------ RMSNorm
+// out[r] = h[src] / sqrt(mean(h[src]^2) + eps) * g, src = gather ? gather[r] : r.
+// With head_w: head_out[r] = sigmoid(head_w . normalized row) (fp32, before rounding).
+template <typename T>
+__global__ void k_rmsnorm(const float* h, int D, const T* g, float eps, T* out, size_t plane,
+                          const int32_t* gather, const float* head_w, float* head_out) {
+  __shared__ float red[kMaxWarps];
+  const int r = blockIdx.x;
+  const int src = gather ? gather[r] : r;
+  const float* x = h + (size_t)src * D;
+  float ss = 0.f;
+  for (int c = threadIdx.x; c < D; c += blockDim.x) ss += x[c] * x[c];
+  ss = block_sum(ss, red);
+  const float inv = rsqrtf(ss / (float)D + eps);
+  float hw = 0.f;
+  for (int c = threadIdx.x; c < D; c += blockDim.x) {
+    const float y = x[c] * inv * to_f32<T>(g[c]);
+    store_act<T>(out, plane, (size_t)r * D + c, y);
+    if (head_w) hw += head_w[c] * y;
+  }
+  if (head_w) {
+    hw = block_sum(hw, red);
+    if (threadIdx.x == 0) head_out[r] = 1.0f / (1.0f + expf(-hw));
+  }
+}
+
+// ------------------------------------------------------------------------------ attention
+// One block per (row, kv head): the G = n_heads / kvh query heads of that kv head attend to
+// the row's visible keys (prefix [0, n_prefix) through the page table, then its tail slots).
+__device__ __forceinline__ const float* key_row(const KvStore& kv, int layer, const RowDesc& rd,
+                                                int t, int kvsel, int head) {
+  if (t < rd.n_prefix) {
+    const int page = kv.page_table[rd.b * kv.max_pages + (t >> kv.page_shift)];
+    return kv.pool + kv_prefix_offset(kv, layer, page < 0 ? 0 : page, kvsel, head,
+                                      t & ((1 << kv.page_shift) - 1));
+  }
+  return kv.tail + kv_tail_offset(kv, layer, kvsel, rd.tail_base + (t - rd.n_prefix), head);
+}
+
+template <typename T>
+__global__ void k_attention(const float* q, KvStore kv, int layer, const RowDesc* rows,
+                            int n_heads, T* out, size_t plane, float scale) {
+  extern __shared__ float sm[];
+  const int r = blockIdx.x, g = blockIdx.y;
+  const RowDesc rd = rows[r];
+  const int hd = kv.hd, G = n_heads / kv.kvh;
+  const int nkeys = rd.n_prefix + rd.n_tail;
+  float* qs = sm;              // [G][hd]
+  float* sc = sm + G * hd;     // [G][nkeys]
+  __shared__ float inv_sum[16];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (int i = threadIdx.x; i < G * hd; i += blockDim.x)
+    qs[i] = q[(size_t)r * n_heads * hd + (size_t)g * G * hd + i] * scale;
+  __syncthreads();
+  for (int t = wid; t < nkeys; t += nw) {
+    const float* kr = key_row(kv, layer, rd, t, 0, g);
+    for (int gg = 0; gg < G; ++gg) {
+      float s = 0.f;
+      for (int e = lane; e < hd; e += 32) s += qs[gg * hd + e] * kr[e];
+      s = warp_sum(s);
+      if (lane == 0) sc[gg * nkeys + t] = s;
+    }
+  }
+  __syncthreads();
+  for (int gg = wid; gg < G; gg += nw) {
+    float m = -INFINITY;
+    for (int t = lane; t < nkeys; t += 32) m = fmaxf(m, sc[gg * nkeys + t]);
+    m = warp_max(m);
+    float z = 0.f;
+    for (int t = lane; t < nkeys; t += 32) {
+      const float p = expf(sc[gg * nkeys + t] - m);
+      sc[gg * nkeys + t] = p;
+      z += p;
+    }
+    z = warp_sum(z);
+    if (lane == 0) inv_sum[gg] = 1.0f / z;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < G * hd; i += blockDim.x) {
+    const int gg = i / hd, e = i % hd;
+    float acc = 0.f;
+    for (int t = 0; t < nkeys; ++t) acc += sc[gg * nkeys + t] * key_row(kv, layer, rd, t, 1, g)[e];
+    store_act<T>(out, plane, (size_t)r * n_heads * hd + (size_t)g * G * hd + i, acc * inv_sum[gg]);
+  }
+}
+
+// ------------------------------------------------------------------------------ row stats
+__global__ void k_row_stats(RowStatsArgs a) {
+  __shared__ unsigned long long redk[kMaxWarps];
+  __shared__ float red[kMaxWarps];
+  __shared__ int bad_s;
+  const int r = blockIdx.x;
+  const float* v = a.logits + (size_t)r * a.V;
+  if (threadIdx.x == 0) bad_s = 0;
+  __syncthreads();
+  unsigned long long best = 0;
+  int bad = 0;
+  for (int i = threadIdx.x; i < a.V; i += blockDim.x) {
+    const float x = v[i];
+    if (!isfinite(x)) bad = 1;
+    const unsigned long long key = argmax_key(x, i);
+    best = key > best ? key : best;
+  }
+  if (bad) atomicOr(&bad_s, 1);
+  best = block_max_u64(best, redk);
+  const int amax = argmax_key_index(best);
+  const float m = v[amax];
+  float z = 0.f;
+  for (int i = threadIdx.x; i < a.V; i += blockDim.x) z += expf(v[i] - m);
+  z = block_sum(z, red);
+  const float lse = m + logf(z);
+  if (threadIdx.x == 0 && bad_s) set_status(a.status, CDSL_ENONFINITE);
+
+  if (a.x_out) {  // draft rollout: greedy token and its log-probability
+    if (threadIdx.x == 0) {
+      a.x_out[r * a.out_stride + a.out_off] = amax;
+      a.logq_out[r * a.out_stride + a.out_off] = m - lse;
+    }
+    return;
+  }
+  if (a.amax && threadIdx.x == 0) a.amax[r] = amax;
+  if (a.dp1 > 0 && threadIdx.x == 0) {
+    const int j = r % a.dp1, bi = r / a.dp1, d = a.dp1 - 1;
+    if (j < d && a.logp) {
+      const int tok = a.next_x[bi * d + j];
+      a.logp[bi * d + j] = v[tok] - lse;
+    }
+  }
+  if (a.topk) {
+    int dst = r;
+    if (a.dst) dst = a.dst[r];
+    if (dst < 0) return;
+    unsigned long long prev = best;
+    if (threadIdx.x == 0) a.topk[dst * a.k] = amax;
+    for (int p = 1; p < a.k; ++p) {
+      unsigned long long cur = 0;
+      for (int i = threadIdx.x; i < a.V; i += blockDim.x) {
+        const unsigned long long key = argmax_key(v[i], i);
+        if (key < prev && key > cur) cur = key;
+      }
+      cur = block_max_u64(cur, redk);
+      if (threadIdx.x == 0) a.topk[dst * a.k + p] = argmax_key_index(cur);
+      prev = cur;
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------ plans
+// Draft call j (1..d): beam rows (b, i) carry c_bi (j = 1) or x_bi,j-1 at position L + j - 1,
+// see the prefix and their own tail slots 0..j-1. Call 1 adds one row per prompt: the pending
+// token L-1 of a fully accepted step, written straight into the draft prefix pages.
+__global__ void k_plan_draft(StepState st, int j, int spb, RowDesc* rows) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  const int nbk = st.B * st.k;
+  if (r < nbk) {
+    const int b = r / st.k;
+    const int L = st.len[b];
+    RowDesc rd;
+    rd.b = b;
+    rd.pos = L + j - 1;
+    rd.token = (j == 1) ? st.roots[r] : st.x[r * st.d + j - 2];
+    rd.n_prefix = L;
+    rd.tail_base = r * spb;
+    rd.n_tail = j;
+    rd.kv_dst = r * spb + j - 1;
+    rd.out_idx = r;
+    rows[r] = rd;
+  } else if (j == 1 && r < nbk + st.B) {
+    const int b = r - nbk;
+    const int L = st.len[b];
+    RowDesc rd;
+    rd.b = b;
+    rd.tail_base = 0;
+    rd.n_tail = 0;
+    rd.out_idx = -1;
+    if (st.pend[b]) {
+      rd.pos = L - 1;
+      rd.token = st.tokens[b * st.lcap + L - 1];
+      rd.n_prefix = L;
+      rd.kv_dst = KV_PREFIX;
+    } else {  // idle row: reads position 0, stores nothing
+      rd.pos = 0;
+      rd.token = 0;
+      rd.n_prefix = 1;
+      rd.kv_dst = KV_NONE;
+    }
+    rows[r] = rd;
+  }
+}
+
+// Verify rows (b, i, j), j = 0..d: token c_bi (j = 0) or x_bi,j at position L + j; they see
+// the prefix and their beam's tail slots 0..j (causal within the beam, nothing across beams).
+__global__ void k_plan_verify(StepState st, RowDesc* rows) {
+  const int dp1 = st.d + 1;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= st.B * st.k * dp1) return;
+  const int bi = r / dp1, j = r % dp1, b = bi / st.k;
+  const int L = st.len[b];
+  RowDesc rd;
+  rd.b = b;
+  rd.pos = L + j;
+  rd.token = (j == 0) ? st.roots[bi] : st.x[bi * st.d + j - 1];
+  rd.n_prefix = L;
+  rd.tail_base = bi * dp1;
+  rd.n_tail = j + 1;
+  rd.kv_dst = r;
+  rd.out_idx = r;
+  rows[r] = rd;
+}
+
+// ------------------------------------------------------------------------------ decision
+__device__ void alloc_pages(const KvStore& kv, int b, int from, int to, int32_t* next_page,
+                            int32_t* status) {
+  if (to <= from) return;
+  for (int p = from >> kv.page_shift; p <= (to - 1) >> kv.page_shift; ++p) {
+    int32_t* e = kv.page_table + b * kv.max_pages + p;
+    if (p >= kv.max_pages) { set_status(status, CDSL_ERANGE); return; }
+    if (*e < 0) {
+      const int id = atomicAdd(next_page, 1);
+      if (id >= kv.n_pages) { set_status(status, CDSL_ERANGE); return; }
+      *e = id;
+    }
+  }
+}
+
+// One warp per prompt, one lane per beam: n_b, rewards, b*, state, emission, page allocation.
+__global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
+  const int b = blockIdx.x, lane = threadIdx.x;
+  const int k = st.k, d = st.d, dp1 = d + 1;
+  if (st.gen[b] >= st.max_new) {
+    if (lane < k) {
+      st.reward[(b * k + lane) * 2] = 0.f;
+      st.reward[(b * k + lane) * 2 + 1] = 0.f;
+      st.n_acc[b * k + lane] = 0;
+    }
+    if (lane < dp1) st.emitted[b * dp1 + lane] = -1;
+    if (lane == 0) { st.beam[b] = -1; st.state[b] = 0; st.n_emit[b] = 0; }
+    return;
+  }
+  float rf = -INFINITY, ra = -INFINITY;
+  int n = 0;
+  if (lane < k) {
+    const int bi = b * k + lane;
+    for (int j = 0; j < d; ++j) {
+      if (st.v_amax[bi * dp1 + j] != st.x[bi * d + j]) break;
+      ++n;
+    }
+    const int root = st.roots[bi];
+    uint32_t cf = st.cov[b], ca = st.cov[b];
+    for (int q = 0; q < st.nk; ++q) {
+      const int kwq = st.kw[b * st.nk + q];
+      bool in_full = (root == kwq), in_acc = (root == kwq);
+      for (int j = 0; j < d; ++j) {
+        const bool hit = st.x[bi * d + j] == kwq;
+        in_full |= hit;
+        in_acc |= hit && (j < n);
+      }
+      if (in_full) cf |= 1u << q;
+      if (in_acc) ca |= 1u << q;
+    }
+    const float covf = (float)__popc(cf) / (float)st.nk;
+    const float cova = (float)__popc(ca) / (float)st.nk;
+    if (st.reward_head) {
+      rf = 0.5f * covf + 0.5f * st.v_head[bi * dp1 + d];
+      ra = 0.5f * cova + 0.5f * st.v_head[bi * dp1 + n];
+    } else {
+      rf = covf;
+      ra = cova;
+    }
+    st.n_acc[bi] = n;
+    st.reward[bi * 2] = rf;
+    st.reward[bi * 2 + 1] = ra;
+  }
+  const unsigned long long key = (lane < k) ? argmax_key(rf, lane) : 0ull;
+  const int bs = argmax_key_index(warp_max_u64(key));   // first beam with the largest r^full
+  const int nb = __shfl_sync(0xffffffffu, n, bs);
+  const float rab = __shfl_sync(0xffffffffu, ra, bs);
+  const bool s1 = (nb >= st.n_min) && (rab >= st.r_t);
+  int cnt = s1 ? 1 + nb : 1;
+  cnt = min(cnt, st.max_new - st.gen[b]);
+  const int bbi = b * k + bs;
+  if (lane < dp1) {
+    int tok = -1;
+    if (lane < cnt) tok = (lane == 0) ? st.roots[bbi] : st.x[bbi * d + lane - 1];
+    st.emitted[b * dp1 + lane] = tok;
+  }
+  if (lane == 0) {
+    st.beam[b] = bs;
+    st.state[b] = s1 ? 1 : (nb < st.n_min ? 2 : 4);
+    st.n_emit[b] = cnt;
+    if (!commit) return;
+    const int L = st.len[b];
+    alloc_pages(tkv, b, L, L + cnt, st.next_page + 0, st.status);
+    alloc_pages(dkv, b, L, L + cnt, st.next_page + 1, st.status);
+  }
+}
+
+// Copy the winner's tail K/V rows 0..cnt-1 to prefix positions L..L+cnt-1.
+__global__ void k_commit_kv(StepState st, KvStore kv, int spb, int is_draft) {
+  const int b = blockIdx.x, layer = blockIdx.y, kvsel = blockIdx.z;
+  int cnt = st.n_emit[b];
+  if (is_draft) cnt = min(cnt, st.d);
+  if (cnt <= 0) return;
+  const int bs = st.beam[b], L = st.len[b];
+  const int per_row = kv.kvh * kv.hd;
+  for (int e = threadIdx.x; e < cnt * per_row; e += blockDim.x) {
+    const int j = e / per_row, rest = e % per_row, head = rest / kv.hd, c = rest % kv.hd;
+    const int pos = L + j;
+    const int page = kv.page_table[b * kv.max_pages + (pos >> kv.page_shift)];
+    if (page < 0) continue;
+    const float* src = kv.tail + kv_tail_offset(kv, layer, kvsel, (b * st.k + bs) * spb + j, head);
+    float* dst = kv.pool + kv_prefix_offset(kv, layer, page, kvsel, head, pos & ((1 << kv.page_shift) - 1));
+    dst[c] = src[c];
+  }
+}
+
+// pfx <- pfx + O, T <- T + O; the next beams are the top-k of the winner's row cnt-1.
+__global__ void k_advance(StepState st) {
+  const int b = blockIdx.x, lane = threadIdx.x;
+  const int k = st.k, d = st.d, dp1 = d + 1;
+  if (b == 0 && lane == 0) {
+    st.counters[0] += 1;       // steps
+    st.counters[1] += d;       // draft forward passes
+    st.counters[2] += 1;       // target forward passes
+  }
+  const int cnt = st.n_emit[b];
+  if (cnt <= 0) return;
+  const int L = st.len[b], bs = st.beam[b];
+  if (lane < cnt) st.tokens[b * st.lcap + L + lane] = st.emitted[b * dp1 + lane];
+  uint32_t bits = 0;
+  if (lane < st.nk) {
+    const int kwq = st.kw[b * st.nk + lane];
+    for (int t = 0; t < cnt; ++t)
+      if (st.emitted[b * dp1 + t] == kwq) bits = 1u << lane;
+  }
+  for (int o = 16; o > 0; o >>= 1) bits |= __shfl_xor_sync(0xffffffffu, bits, o);
+  const int root_row = (b * k + bs) * dp1 + cnt - 1;
+  if (lane < k) st.roots[b * k + lane] = st.v_topk[root_row * k + lane];
+  if (lane == 0) {
+    st.cov[b] |= bits;
+    st.len[b] = L + cnt;
+    st.gen[b] += cnt;
+    st.pend[b] = (cnt == dp1) ? 1 : 0;
+    atomicAdd((unsigned long long*)&st.counters[3], (unsigned long long)cnt);
+    if (st.state[b] == 1) atomicAdd((unsigned long long*)&st.counters[4], 1ull);
+    atomicAdd((unsigned long long*)&st.counters[5], 1ull);
+  }
+}
+
+__global__ void k_rope_table(float2* table, int n_pos, int hd, double theta) {
+  const int half = hd / 2;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n_pos * half) return;
+  const int pos = i / half, m = i % half;
+  const double ang = (double)pos * pow(theta, -2.0 * m / hd);
+  double s, c;
+  sincos(ang, &s, &c);
+  table[i] = make_float2((float)c, (float)s);
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------------------ launchers
+#define DISPATCH(dtype, ...)                                   \
+  do {                                                         \
+    if ((dtype) == CDSL_DTYPE_BF16) {                          \
+      using T = __nv_bfloat16;                                 \
+      __VA_ARGS__;                                             \
+    } else {                                                   \
+      using T = float;                                         \
+      __VA_ARGS__;                                             \
+    }                                                          \
+  } while (0)
+
+void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int D, float* h,
+                  cudaStream_t s) {
+  DISPATCH(dtype, k_embed<T><<<R, 256, 0, s>>>(rows, (const T*)embed, D, h));
+}
+
+void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
+                    void* out, size_t plane, const int32_t* gather, const float* head_w,
+                    float* head_out, cudaStream_t s) {
+  DISPATCH(dtype, k_rmsnorm<T><<<R, 256, 0, s>>>(h, D, (const T*)gain, eps, (T*)out, plane,
+                                                 gather, head_w, head_out));
+}
+
+void launch_attention(int dtype, const float* q, KvStore kv, int layer, const RowDesc* rows,
+                      int R, int n_heads, int max_keys, void* out, size_t plane,
+                      int32_t* status, cudaStream_t s) {
+  const int G = n_heads / kv.kvh;
+  const size_t smem = sizeof(float) * ((size_t)G * kv.hd + (size_t)G * max_keys);
+  const float scale = 1.0f / sqrtf((float)kv.hd);
+  dim3 grid(R, kv.kvh);
+  DISPATCH(dtype, {
+    static int configured = 0;
+    if (smem > 48 * 1024 && configured < (int)smem) {
+      cudaFuncSetAttribute(k_attention<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      configured = (int)smem;
+    }
+    k_attention<T><<<grid, 128, smem, s>>>(q, kv, layer, rows, n_heads, (T*)out, plane, scale);
+  });
+  (void)status;
+}
+
+void launch_row_stats(const RowStatsArgs& a, cudaStream_t s) {
+  k_row_stats<<<a.R, 512, 0, s>>>(a);
+}
+
+void launch_plan_draft(const StepState& st, int j, int spb, RowDesc* rows, cudaStream_t s) {
+  const int n = st.B * st.k + (j == 1 ? st.B : 0);
+  k_plan_draft<<<(n + 127) / 128, 128, 0, s>>>(st, j, spb, rows);
+}
+
+void launch_plan_verify(const StepState& st, RowDesc* rows, cudaStream_t s) {
+  const int n = st.B * st.k * (st.d + 1);
+  k_plan_verify<<<(n + 127) / 128, 128, 0, s>>>(st, rows);
+}
+
+void launch_select(const StepState& st, KvStore tkv, KvStore dkv, int commit, cudaStream_t s) {
+  k_select<<<st.B, 32, 0, s>>>(st, tkv, dkv, commit);
+}
+
+void launch_commit_kv(const StepState& st, KvStore kv, int spb, int is_draft, cudaStream_t s) {
+  dim3 grid(st.B, kv.n_layers, 2);
+  k_commit_kv<<<grid, 256, 0, s>>>(st, kv, spb, is_draft);
+}
+
+void launch_advance(const StepState& st, cudaStream_t s) { k_advance<<<st.B, 32, 0, s>>>(st); }
+
+void launch_rope_table(float2* table, int n_pos, int hd, float theta, cudaStream_t s) {
+  const int n = n_pos * (hd / 2);
+  k_rope_table<<<(n + 255) / 256, 256, 0, s>>>(table, n_pos, hd, (double)theta);
+}
+
+}  // namespace cdsl

@@ -1,0 +1,79 @@
+// kernels.h -- host launchers of the CDSL step kernels (declarations).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+#include "gemm.cuh"
+
+namespace cdsl {
+
+// Per-prompt decoding state on the device (all pointers into the workspace).
+struct StepState {
+  int32_t B, k, d, nk, max_new, lcap, n_min, reward_head;
+  float r_t;
+  int32_t* len;        // [B] committed prefix length L (target; draft up to the pending row)
+  int32_t* pend;       // [B] 1: the draft still lacks the KV of token L-1
+  int32_t* gen;        // [B] tokens generated (len(T))
+  int32_t* tokens;     // [B, lcap]
+  int32_t* roots;      // [B, k]
+  int32_t* kw;         // [B, nk]
+  uint32_t* cov;       // [B] keyword bits already covered by T
+  int32_t* x;          // [B, k, d] drafted tokens
+  float* logq;         // [B, k, d]
+  int32_t* v_amax;     // [B*k*(d+1)] verify row argmax
+  float* v_logp;       // [B, k, d] log p_j(x_j)
+  int32_t* v_topk;     // [B*k*(d+1), k]
+  float* v_head;       // [B*k*(d+1)] sigmoid(w . h)
+  int32_t* n_acc;      // [B, k]
+  float* reward;       // [B, k, 2]
+  int32_t* beam;       // [B]
+  int32_t* state;      // [B]
+  int32_t* emitted;    // [B, d+1]
+  int32_t* n_emit;     // [B]
+  int32_t* next_page;  // [2] bump allocators (target, draft)
+  int32_t* status;     // device status word
+  long long* counters; // [8]
+};
+
+// elementwise / row kernels (T = float or __nv_bfloat16, the model dtype)
+void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int D, float* h,
+                  cudaStream_t s);
+// out: GEMM-input activations (store_act format, hi/lo planes `plane` elements apart)
+void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
+                    void* out, size_t plane, const int32_t* gather, const float* head_w,
+                    float* head_out, cudaStream_t s);
+void launch_attention(int dtype, const float* q, KvStore kv, int layer, const RowDesc* rows,
+                      int R, int n_heads, int max_keys, void* out, size_t plane,
+                      int32_t* status, cudaStream_t s);
+// Row statistics of logits rows: argmax (lower id on ties), log-sum-exp, top-k, log p.
+//   draft mode  (dp1 == 0): x[r*out_stride + out_off] = argmax, logq[...] = log q(argmax)
+//   verify mode (dp1 == d+1): amax[r], topk[r, k], logp of the next drafted token
+//   roots mode  (topk only): topk of row r written to row dst[r] of topk
+struct RowStatsArgs {
+  const float* logits; int32_t R, V, k;
+  int32_t dp1;                 // d+1 in verify mode, else 0
+  const int32_t* next_x;       // verify: drafted tokens [B,k,d]
+  int32_t* amax; float* logp;  // verify: [R], [B,k,d]
+  int32_t* topk;               // verify / roots: [R or B, k]
+  const int32_t* dst;          // roots: destination row per logits row
+  int32_t* x_out; float* logq_out; int32_t out_stride, out_off;  // draft
+  int32_t* status;
+};
+void launch_row_stats(const RowStatsArgs& a, cudaStream_t s);
+
+void launch_gemm_simt(int dtype, const GemmArgs& a, cudaStream_t s);
+
+// plans and the decision
+void launch_plan_draft(const StepState& st, int j, int tail_slots_per_beam, RowDesc* rows,
+                       cudaStream_t s);
+void launch_plan_verify(const StepState& st, RowDesc* rows, cudaStream_t s);
+// commit = 0: decide only (n_b, rewards, b*, state, emission); 1: also allocate KV pages
+void launch_select(const StepState& st, KvStore tkv, KvStore dkv, int commit, cudaStream_t s);
+void launch_commit_kv(const StepState& st, KvStore kv, int slots_per_beam, int is_draft,
+                      cudaStream_t s);
+void launch_advance(const StepState& st, cudaStream_t s);
+void launch_rope_table(float2* table, int n_pos, int hd, float theta, cudaStream_t s);
+
+}  // namespace cdsl

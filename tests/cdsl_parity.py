@@ -1,0 +1,152 @@
+"""Helpers that run the CUDA path and the oracle side by side on the same seeded inputs."""
+from __future__ import annotations
+
+import dataclasses
+from typing import Dict, List, Optional
+
+import numpy as np
+
+import synth
+import oracle
+
+
+@dataclasses.dataclass
+class Setup:
+    wl: synth.Workload
+    t_host: Dict[str, np.ndarray]
+    d_host: Dict[str, np.ndarray]
+    prompts: np.ndarray
+    lens: List[int]
+    keywords: np.ndarray
+    w_head: np.ndarray
+
+
+def make_setup(wl: synth.Workload, lens=None, keywords=None, draft_equals_target=False,
+               host=True) -> Setup:
+    t = synth.model_weights(wl, "target", device="host") if host else None
+    d = t if draft_equals_target else (synth.model_weights(wl, "draft", device="host") if host else None)
+    p = synth.prompts(wl)
+    lens = list(lens) if lens is not None else [wl.prompt_len] * wl.batch
+    kw = synth.keywords(wl) if keywords is None else np.asarray(keywords, dtype=np.int32)
+    return Setup(wl, t, d, p, lens, kw, synth.reward_head(wl))
+
+
+def run_params(wl: synth.Workload) -> oracle.RunParams:
+    return oracle.RunParams(k=wl.k, d=wl.d, a_t=wl.a_t, r_t=wl.r_t, max_new=wl.max_new,
+                            composite_reward=wl.reward_head)
+
+
+def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0):
+    import torch
+    import paper_2412_10418_gb300 as cdsl
+
+    wl = s.wl
+    if torch_weights is None:
+        tw = synth.to_torch(s.t_host, wl.dtype)
+        dw = tw if s.d_host is s.t_host else synth.to_torch(s.d_host, wl.dtype)
+    else:
+        tw, dw = torch_weights
+    dshape = wl.target if s.d_host is s.t_host else wl.draft
+    order_t = [tw[n] for n, _ in wl.target.weight_specs()]
+    order_d = [dw[n] for n, _ in dshape.weight_specs()]
+    head = torch.from_numpy(s.w_head).cuda() if wl.reward_head else None
+    eng = cdsl.Engine(wl.target, dshape, wl.dtype, order_t, order_d, batch=wl.batch, k=wl.k,
+                      d=wl.d, max_prompt=wl.prompt_len, max_new=wl.max_new,
+                      n_keywords=s.keywords.shape[1], a_t=wl.a_t, r_t=wl.r_t, reward_head=head,
+                      page_size=page_size, max_chunk=max_chunk)
+    eng.prefill(torch.from_numpy(s.prompts), s.lens, torch.from_numpy(s.keywords))
+    return eng
+
+
+def oracle_models(s: Setup):
+    wl = s.wl
+    tgt = oracle.Transformer(wl.target, s.t_host)
+    drf = tgt if s.d_host is s.t_host else oracle.Transformer(wl.draft, s.d_host)
+    return tgt, drf
+
+
+def oracle_prefill(s: Setup, tgt, drf):
+    states = []
+    for b in range(s.wl.batch):
+        p = s.prompts[b, :s.lens[b]][None]
+        states += oracle.prefill(tgt, drf, p, s.keywords[b:b + 1])
+    return states
+
+
+def gpu_step_outputs(eng, with_logits=True):
+    """One step through the three separate calls; returns numpy copies of every output."""
+    import torch
+
+    lg = None
+    if with_logits:
+        lg = torch.empty((eng.B, eng.k, eng.d + 1, eng.V), dtype=torch.float32, device="cuda")
+    eng.lookahead()
+    eng.verify(lg)
+    eng.select()
+    eng.stream.synchronize()
+    out = {n: getattr(eng, n).cpu().numpy() for n in
+           ("roots", "draft_tok", "logq", "logp", "argmax", "n_accept", "beam", "state",
+            "emitted", "n_emitted", "reward")}
+    out["logits"] = lg.cpu().numpy() if with_logits else None
+    return out
+
+
+def compare_step(g, recs, tol, tol_r, report):
+    """Element-wise comparison of one GPU step with the oracle's (after near-tie resolution).
+
+    Returns the largest absolute differences seen; raises AssertionError on any mismatch."""
+    worst = dict(logits=0.0, logq=0.0, logp=0.0, reward=0.0)
+    for b, rec in enumerate(recs):
+        if not rec.active:
+            assert g["n_emitted"][b] == 0, f"prompt {b}: finished but emitted"
+            continue
+        where = f"prompt {b}"
+        assert np.array_equal(g["roots"][b], rec.roots), f"{where}: roots {g['roots'][b]} vs {rec.roots}"
+        assert np.array_equal(g["draft_tok"][b], rec.x), f"{where}: draft tokens"
+        worst["logq"] = max(worst["logq"], float(np.max(np.abs(g["logq"][b] - rec.logq))))
+        if g["logits"] is not None:
+            worst["logits"] = max(worst["logits"], float(np.max(np.abs(g["logits"][b] - rec.vlogits))))
+        assert np.array_equal(g["argmax"][b], rec.argmax), f"{where}: verify argmax"
+        worst["logp"] = max(worst["logp"], float(np.max(np.abs(g["logp"][b] - rec.logp))))
+        assert np.array_equal(g["n_accept"][b], rec.n), f"{where}: n {g['n_accept'][b]} vs {rec.n}"
+        rw = np.stack([rec.r_full, rec.r_acc], axis=-1)
+        worst["reward"] = max(worst["reward"], float(np.max(np.abs(g["reward"][b] - rw))))
+        assert g["beam"][b] == rec.beam, f"{where}: beam {g['beam'][b]} vs {rec.beam}"
+        assert g["state"][b] == rec.state, f"{where}: state {g['state'][b]} vs {rec.state}"
+        ne = int(g["n_emitted"][b])
+        assert g["emitted"][b][:ne].tolist() == rec.emitted, f"{where}: emitted"
+        assert np.all(g["emitted"][b][ne:] == -1)
+    for key, lim in (("logits", tol), ("logq", tol), ("logp", tol), ("reward", tol_r)):
+        assert worst[key] <= lim, f"{key}: max |diff| {worst[key]:.3g} > {lim}"
+        report.setdefault(key, 0.0)
+        report[key] = max(report[key], worst[key])
+    return worst
+
+
+def decider_from(g, tol, tol_r):
+    other = {"roots": g["roots"], "x": g["draft_tok"], "argmax": g["argmax"],
+             "beam": g["beam"], "s1": g["state"] == oracle.S1}
+    return oracle.Decider(other=other, tol=tol, tol_r=tol_r)
+
+
+def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_size=16,
+               max_chunk=0):
+    """Step the GPU and the oracle together; every step is compared element by element."""
+    eng = eng or make_engine(s, page_size=page_size, max_chunk=max_chunk)
+    tgt, drf = oracle_models(s)
+    states = oracle_prefill(s, tgt, drf)
+    run = run_params(s.wl)
+    report: Dict[str, float] = {}
+    adopted = []
+    n_steps = 0
+    for _ in range(steps):
+        if all(len(st.T) >= run.max_new for st in states):
+            break
+        g = gpu_step_outputs(eng)
+        dec = decider_from(g, tol, tol_r)
+        recs = oracle.cdsl_k_step(tgt, drf, states, run, s.w_head, dec)
+        compare_step(g, recs, tol, tol_r, report)
+        adopted += dec.adopted
+        n_steps += 1
+    assert eng.status() == 0
+    return eng, states, report, adopted, n_steps

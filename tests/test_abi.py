@@ -1,0 +1,126 @@
+"""The C-ABI library loads, exports every symbol include/cdsl.h declares, and validates its
+host-side arguments (no GPU needed: these calls launch nothing)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def cdsl():
+    from paper_2412_10418_gb300 import build as b
+    b.build()
+    import paper_2412_10418_gb300 as pkg
+    return pkg
+
+
+def declared_symbols():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if h.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", h)).read()
+            names |= set(re.findall(r"CDSL_API[^;(]*?\b(cdsl_\w+)\s*\(", src))
+    return names
+
+
+def test_exports_every_declared_symbol(cdsl):
+    names = declared_symbols()
+    assert {"cdsl_init", "cdsl_lookahead", "cdsl_verify", "cdsl_select", "cdsl_step"} <= names
+    lib = ctypes.CDLL(cdsl.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), n
+    # the binding declares exactly the exported entry points
+    assert set(cdsl.EXPORTS) <= names
+
+
+def cfgs(cdsl, wl=synth.TINY, **run_kw):
+    t = cdsl.model_cfg(wl.target, wl.dtype)
+    d = cdsl.model_cfg(wl.draft, wl.dtype)
+    kw = dict(batch=wl.batch, k=wl.k, d=wl.d, max_prompt=wl.prompt_len, max_new=wl.max_new,
+              n_keywords=wl.n_keywords, a_t=wl.a_t, r_t=wl.r_t, reward_head=wl.reward_head)
+    kw.update(run_kw)
+    return t, d, cdsl.run_cfg(**kw)
+
+
+def test_num_weights(cdsl):
+    t, d, _ = cfgs(cdsl)
+    assert cdsl.cdsl_num_weights(t) == len(synth.TINY.target.weight_specs())
+    assert cdsl.cdsl_num_weights(d) == len(synth.TINY.draft.weight_specs())
+
+
+def test_workspace_size_grows_with_work(cdsl):
+    t, d, r = cfgs(cdsl)
+    n1 = cdsl.cdsl_workspace_size(t, d, r)
+    t2, d2, r2 = cfgs(cdsl, batch=4, k=8, d=6, max_new=64)
+    n2 = cdsl.cdsl_workspace_size(t2, d2, r2)
+    assert 0 < n1 < n2 and n1 % 256 == 0
+    # 7B-shaped target: the KV pool alone is 32 layers * 2 * 8 * 128 * 2 B per position
+    wl = synth.SEVEN_B
+    t7, d7, r7 = cfgs(cdsl, wl)
+    n7 = cdsl.cdsl_workspace_size(t7, d7, r7)
+    assert n7 > (wl.prompt_len + wl.max_new) * 32 * 2 * 8 * 128 * 2
+
+
+@pytest.mark.parametrize("field,value,msg", [
+    ("head_dim", 96, "head_dim"),
+    ("n_kv_heads", 3, "n_kv_heads"),
+    ("dtype", 7, "dtype"),
+    ("d_model", 100, "d_model"),
+])
+def test_bad_model_config(cdsl, field, value, msg):
+    t, d, r = cfgs(cdsl)
+    setattr(t, field, value)
+    with pytest.raises(cdsl.CdslError) as e:
+        cdsl.cdsl_workspace_size(t, d, r)
+    assert e.value.code == 1 and msg in str(e.value)
+
+
+@pytest.mark.parametrize("field,value", [("k", 0), ("k", 17), ("d", 0), ("n_keywords", 33),
+                                         ("page_size", 48), ("batch", 0)])
+def test_bad_run_config(cdsl, field, value):
+    t, d, r = cfgs(cdsl)
+    setattr(r, field, value)
+    with pytest.raises(cdsl.CdslError) as e:
+        cdsl.cdsl_workspace_size(t, d, r)
+    assert e.value.code == 1
+
+
+def test_vocab_and_dtype_must_match(cdsl):
+    t, d, r = cfgs(cdsl)
+    d.vocab = 256
+    with pytest.raises(cdsl.CdslError, match="vocab"):
+        cdsl.cdsl_workspace_size(t, d, r)
+    t, d, r = cfgs(cdsl)
+    d.dtype = 1
+    with pytest.raises(cdsl.CdslError, match="dtype"):
+        cdsl.cdsl_workspace_size(t, d, r)
+
+
+def test_init_rejects_before_touching_the_device(cdsl):
+    """cdsl_init validates everything on the host first: NULL weights, NULL workspace,
+    a missing reward head."""
+    t, d, r = cfgs(cdsl)
+    lib = cdsl.lib()
+    ctx = ctypes.c_void_p(0)
+    nt = cdsl.cdsl_num_weights(t)
+    nd = cdsl.cdsl_num_weights(d)
+    tw = (ctypes.c_void_p * nt)(*([None] * nt))
+    dw = (ctypes.c_void_p * nd)(*([None] * nd))
+    code = lib.cdsl_init(ctypes.byref(t), tw, ctypes.byref(d), dw, ctypes.byref(r), None,
+                         None, 0, None, ctypes.byref(ctx))
+    assert code == 1 and "workspace" in cdsl.cdsl_last_error(None)
+    fake = (ctypes.c_void_p * nt)(*([4096] * nt))
+    fake_d = (ctypes.c_void_p * nd)(*([4096] * nd))
+    code = lib.cdsl_init(ctypes.byref(t), tw, ctypes.byref(d), fake_d, ctypes.byref(r), None,
+                         1 << 20, 1 << 30, None, ctypes.byref(ctx))
+    assert code == 1 and "weight" in cdsl.cdsl_last_error(None)
+    r.reward_head = 1
+    code = lib.cdsl_init(ctypes.byref(t), fake, ctypes.byref(d), fake_d, ctypes.byref(r), None,
+                         1 << 20, 1 << 30, None, ctypes.byref(ctx))
+    assert code == 1 and "reward" in cdsl.cdsl_last_error(None)
+    assert ctx.value is None

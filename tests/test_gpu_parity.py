@@ -1,0 +1,119 @@
+"""CUDA path vs the oracle, element by element, through the C ABI.
+
+Tolerances (stated by the target of this work for the two precisions): logits / log-probs
+|diff| <= 1e-4 for the float32 workload, <= 2e-2 for bf16 weights with fp32 accumulation.
+Token ids, n_b, b*, the state and the emitted tokens must be identical; at a near tie (the
+oracle's own margin below the tolerance) the oracle adopts the CUDA path's choice and the run
+continues along it."""
+import numpy as np
+import pytest
+
+import synth
+import oracle
+from cdsl_parity import (compare_step, decider_from, gpu_step_outputs, make_engine, make_setup,
+                         oracle_models, oracle_prefill, run_params, run_parity)
+
+pytestmark = pytest.mark.gpu
+
+TOL32 = 1e-4
+TOL16 = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2412_10418_gb300 import build
+    build.build()
+
+
+def tokens_match(eng, states):
+    t, n = eng.tokens()
+    t, n = t.cpu().numpy(), n.cpu().numpy()
+    for b, st in enumerate(states):
+        want = st.prompt + st.T
+        assert n[b] == len(want)
+        assert t[b, :n[b]].tolist() == want
+
+
+def test_tiny_fp32_full_run():
+    s = make_setup(synth.TINY)
+    eng, states, rep, adopted, n = run_parity(s, steps=40, tol=TOL32, tol_r=TOL32)
+    assert all(len(st.T) == synth.TINY.max_new for st in states)
+    tokens_match(eng, states)
+    c = eng.counters()
+    assert c[0] == n and c[3] == synth.TINY.max_new
+
+
+def greedy_chain(tgt, prompt, n):
+    toks = list(prompt)
+    for _ in range(n):
+        toks.append(int(np.argmax(tgt.forward_full(toks)[0][-1])))
+    return toks[len(prompt):]
+
+
+def test_tiny_forced_acceptance_s1_and_pending_rows():
+    """Draft := target: every lookahead is accepted (n = d). Keywords taken from the target's
+    greedy continuation make the reward clear r_t, so steps are S1 and emit d+1 tokens; the
+    next step's first draft call must then fill the draft KV of the last drafted token."""
+    wl = synth.scaled(synth.TINY, draft=synth.TINY.target, max_new=24)
+    s = make_setup(wl, draft_equals_target=True)
+    tgt = oracle.Transformer(wl.target, s.t_host)
+    chain = greedy_chain(tgt, s.prompts[0].tolist(), 12)
+    s.keywords = np.array([[chain[2], chain[7], chain[11]]], dtype=np.int32)
+    eng, states, rep, adopted, n = run_parity(s, steps=30, tol=TOL32, tol_r=TOL32)
+    tokens_match(eng, states)
+    c = eng.counters()
+    assert c[4] >= 2, f"expected S1 steps, counters {c}"
+    assert c[3] == wl.max_new
+
+
+def test_ragged_batch_small_pages():
+    wl = synth.scaled(synth.TINY, batch=3, prompt_len=40, max_new=12)
+    s = make_setup(wl, lens=[40, 17, 33])
+    eng, states, rep, adopted, n = run_parity(s, steps=20, tol=TOL32, tol_r=TOL32, page_size=16,
+                                              max_chunk=24)
+    tokens_match(eng, states)
+
+
+@pytest.mark.parametrize("k,d", [(1, 1), (2, 3), (16, 2)])
+def test_beam_and_lookahead_extremes(k, d):
+    wl = synth.scaled(synth.TINY, k=k, d=d, max_new=7)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=10, tol=TOL32, tol_r=TOL32)
+    tokens_match(eng, states)
+
+
+def test_graph_step_equals_separate_calls():
+    import torch
+    wl = synth.scaled(synth.TINY, batch=2, max_new=12)
+    s = make_setup(wl)
+    a = make_engine(s)
+    b = make_engine(s)
+    for _ in range(12):
+        a.step()
+        b.lookahead(); b.verify(); b.select()
+    ta, na = a.tokens()
+    tb, nb = b.tokens()
+    assert torch.equal(na, nb) and torch.equal(ta, tb)
+    assert a.counters()[:6] == b.counters()[:6] and a.counters()[6] > 0
+    assert int(na[0]) == wl.prompt_len + wl.max_new
+
+
+def test_small_bf16_parity():
+    s = make_setup(synth.SMALL)
+    eng, states, rep, adopted, n = run_parity(s, steps=4, tol=TOL16, tol_r=TOL16)
+    assert n == 4
+    print("max |diff|:", rep, "near ties adopted:", len(adopted))
+
+
+def test_nonfinite_logits_are_flagged():
+    """A NaN planted in the input (an embedding row the prompt uses) is reported through the
+    device status word as CDSL_ENONFINITE; nothing faults."""
+    import torch
+    wl = synth.scaled(synth.TINY, max_new=2)
+    s = make_setup(wl)
+    tw = synth.to_torch(s.t_host, wl.dtype)
+    dw = synth.to_torch(s.d_host, wl.dtype)
+    tw["embed"][int(s.prompts[0, 5])] = float("nan")
+    eng = make_engine(s, torch_weights=(tw, dw))
+    eng.lookahead(); eng.verify(); eng.select()
+    assert eng.status() == 5
