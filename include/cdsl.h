@@ -173,7 +173,8 @@ CDSL_API int32_t cdsl_get_counters(cdsl_ctx* ctx, int64_t* h_counters);
  * cdsl_get_profile synchronizes the stream and returns, for GEMM implementation `impl`
  * (0 = CUDA-core tiled GEMM, 1 = weight-streaming GEMV, 2 = tcgen05 tensor-core GEMM),
  * h_out[4] = {launches, total milliseconds, algorithmic bytes (weights read once, activations
- * read, outputs written), flops}; then it clears the record. */
+ * read, outputs written), flops} over the launches recorded since cdsl_profile last enabled
+ * or disabled timing (each call of cdsl_profile clears the record). */
 CDSL_API int32_t cdsl_profile(cdsl_ctx* ctx, int32_t enable);
 CDSL_API int32_t cdsl_get_profile(cdsl_ctx* ctx, int32_t impl, double* h_out);
 

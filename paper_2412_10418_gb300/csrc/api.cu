@@ -2,6 +2,7 @@
 // draft and target models, and the CDSL-k step (lookahead, verify, select) on one stream.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <array>
 #include <cstdio>
 #include <cstring>
@@ -69,6 +70,8 @@ struct cdsl_ctx {
   RowDesc* rows_p = nullptr;
   int32_t* lm_gather = nullptr;
   int32_t* lm_dst = nullptr;
+  float* gemv_part = nullptr;   // split-K partial tiles of the weight-streaming GEMM
+  int32_t* gemv_cnt = nullptr;  // per-tile arrival counters
   StepState st{};
   size_t ws_total = 0;
   int phase = PH_NEW;
@@ -196,6 +199,21 @@ size_t carve(cdsl_ctx* c, void* base) {
   c->rows_p = cv.take<RowDesc>(c->R_p);
   c->lm_gather = cv.take<int32_t>(c->R_p);
   c->lm_dst = cv.take<int32_t>(c->R_p);
+  {  // split-K scratch for the weight-streaming GEMM: the largest projection of either model
+    size_t part = 0, tiles = 0;
+    for (const cdsl_model_cfg* m : {&c->tcfg, &c->dcfg}) {
+      const int D = m->d_model, QH = m->n_heads * m->head_dim, KVH = m->n_kv_heads * m->head_dim;
+      const int shapes[5][2] = {{D, QH + 2 * KVH}, {QH, D}, {D, (m->d_ffn + 63) / 64 * 128},
+                                {m->d_ffn, D}, {D, m->vocab}};
+      for (const auto& sh : shapes) {
+        const GemvPlan p = plan_gemv(sh[0], sh[1], kPlanSMs);
+        part = std::max(part, (size_t)p.splits * 8 * p.tiles * 128);
+        tiles = std::max(tiles, (size_t)p.tiles);
+      }
+    }
+    c->gemv_part = cv.take<float>(part);
+    c->gemv_cnt = cv.take<int32_t>(tiles);
+  }
   StepState& s = c->st;
   s.B = B; s.k = k; s.d = d; s.nk = c->nk; s.max_new = c->run.max_new; s.lcap = c->lcap;
   s.reward_head = c->run.reward_head;
@@ -247,7 +265,7 @@ double gemm_bytes(const cdsl_ctx* c, const GemmArgs& a, double* flops) {
 }
 
 void gemm(cdsl_ctx* c, const GemmArgs& a) {
-  const int impl = 0;
+  const int impl = (c->dtype == CDSL_DTYPE_BF16 && a.R <= 8) ? 1 : 0;
   size_t ev = 0;
   if (c->profiling) {
     while (c->ev_pool.size() < c->ev_used + 2) {
@@ -259,7 +277,10 @@ void gemm(cdsl_ctx* c, const GemmArgs& a) {
     c->ev_used += 2;
     cudaEventRecord(c->ev_pool[ev], c->stream);
   }
-  launch_gemm_simt(c->dtype, a, c->stream);
+  if (impl == 1)
+    launch_gemv(a, plan_gemv(a.K, a.n_virtual, kPlanSMs), c->gemv_part, c->gemv_cnt, c->stream);
+  else
+    launch_gemm_simt(c->dtype, a, c->stream);
   if (c->profiling) {
     cudaEventRecord(c->ev_pool[ev + 1], c->stream);
     double fl = 0;
@@ -682,8 +703,6 @@ int32_t cdsl_get_profile(cdsl_ctx* c, int32_t impl, double* h_out) {
     n += 1; ms += t; by += r.bytes; fl += r.flops;
   }
   h_out[0] = n; h_out[1] = ms; h_out[2] = by; h_out[3] = fl;
-  c->ev_used = 0;
-  c->prof.clear();
   return cuda_check(c, "cdsl_get_profile");
 }
 

@@ -65,6 +65,14 @@ void launch_row_stats(const RowStatsArgs& a, cudaStream_t s);
 
 void launch_gemm_simt(int dtype, const GemmArgs& a, cudaStream_t s);
 
+// Weight-streaming GEMM for R <= 8 activation rows (bf16 weights), split-K over `splits`
+// slices of k_split elements. Scratch: part [splits][8][tiles][128] floats and one arrival
+// counter per tile (zero between launches).
+struct GemvPlan { int splits, k_split, tiles; };
+constexpr int kPlanSMs = 152;  // GB300: split-K is planned for this many SMs
+GemvPlan plan_gemv(int K, int n_virtual, int n_sm);
+void launch_gemv(const GemmArgs& a, const GemvPlan& p, float* part, int* tile_cnt, cudaStream_t s);
+
 // plans and the decision
 void launch_plan_draft(const StepState& st, int j, int tail_slots_per_beam, RowDesc* rows,
                        cudaStream_t s);

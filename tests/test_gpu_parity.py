@@ -105,6 +105,29 @@ def test_small_bf16_parity():
     print("max |diff|:", rep, "near ties adopted:", len(adopted))
 
 
+@pytest.mark.parametrize("batch,k", [(1, 4), (2, 2), (1, 8)])
+def test_small_bf16_few_rows(batch, k):
+    """Draft calls with B*k (+B) <= 8 rows take the weight-streaming GEMM (split-K)."""
+    wl = synth.scaled(synth.SMALL, batch=batch, k=k, max_new=10)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=4, tol=TOL16, tol_r=TOL16)
+    tokens_match(eng, states)
+    print("few rows", batch, k, "max |diff|:", rep)
+
+
+def test_small_bf16_forced_acceptance():
+    """bf16, draft := target, B = 1: full acceptance and S1 emissions through the
+    weight-streaming path, including the pending draft row of the next step."""
+    wl = synth.scaled(synth.SMALL, batch=1, draft=synth.SMALL.target, max_new=16, n_keywords=3)
+    s = make_setup(wl, draft_equals_target=True)
+    tgt = oracle.Transformer(wl.target, s.t_host)
+    chain = greedy_chain(tgt, s.prompts[0].tolist(), 8)
+    s.keywords = np.array([[chain[1], chain[5], chain[7]]], dtype=np.int32)
+    eng, states, rep, adopted, n = run_parity(s, steps=8, tol=TOL16, tol_r=TOL16)
+    tokens_match(eng, states)
+    assert eng.counters()[4] >= 1
+
+
 def test_nonfinite_logits_are_flagged():
     """A NaN planted in the input (an embedding row the prompt uses) is reported through the
     device status word as CDSL_ENONFINITE; nothing faults."""
