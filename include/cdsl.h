@@ -182,8 +182,27 @@ CDSL_API int32_t cdsl_get_profile(cdsl_ctx* ctx, int32_t impl, double* h_out);
  * device-side error was latched) in *h_device_status. Clears nothing. */
 CDSL_API int32_t cdsl_get_status(cdsl_ctx* ctx, int32_t* h_device_status);
 
+/* Weight-streaming GEMM that allocates nothing (the paper has no counterpart; it serves
+ * callers of this library that cannot allocate device memory: code running while a stream
+ * is captured in global mode, where cudaMalloc is an error; host frameworks whose own
+ * allocator holds the GPU's memory; latency-critical loops that must not block on the
+ * allocator). y[R, N] = x[R, K] W^T, fp32 accumulation, computed by the split-K kernel of
+ * the draft calls: d_w [N, K] bfloat16 row-major, d_x [R, K] float32, d_y [R, N] float32,
+ * all device pointers, 16-byte aligned; stream is a cudaStream_t (NULL: legacy stream).
+ * Limits: 1 <= R <= 8, 8 <= K <= 8192 with K % 8 == 0, 1 <= N <= 32768; anything beyond
+ * them returns CDSL_EINVAL without launching. Its scratch (split-K partials, arrival counters
+ * and the hi/lo activation planes, 8.3 MiB) is one fixed array inside the library that every
+ * GPU loading the library holds until the process exits; no call allocates or frees memory.
+ * The first call on a device looks up that array's address (and clears its counters) with
+ * the device current, so make that first call before any stream capture. Every call reuses
+ * the same array: calls that overlap on a GPU (other streams or threads) race, and the caller
+ * must order them. Asynchronous on `stream`; errors via cdsl_last_error(NULL). */
+CDSL_API int32_t cdsl_gemv_noalloc(const void* d_w, int32_t N, int32_t K, const float* d_x,
+                                   int32_t R, float* d_y, void* stream);
+
 /* Message of the last error on this context (never NULL; "" when none). With ctx == NULL,
- * the message of the last failed cdsl_init on this thread. */
+ * the message of the last failed context-free call (cdsl_init, cdsl_workspace_size,
+ * cdsl_gemv_noalloc) on this thread. */
 CDSL_API const char* cdsl_last_error(const cdsl_ctx* ctx);
 
 /* Release the context's host metadata and CUDA graph. Does not free borrowed memory. */

@@ -64,6 +64,7 @@ EXPORTS = {
     "cdsl_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_int32)]),
     "cdsl_profile": (_I, [_P, _I]),
     "cdsl_get_profile": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double)]),
+    "cdsl_gemv_noalloc": (_I, [_P, _I, _I, _P, _I, _P, _P]),
     "cdsl_last_error": (ctypes.c_char_p, [_P]),
     "cdsl_destroy": (None, [_P]),
 }
@@ -190,6 +191,14 @@ def cdsl_get_profile(ctx, impl: int):
     out = (ctypes.c_double * 4)()
     _check(lib().cdsl_get_profile(ctx, impl, out), ctx)
     return dict(launches=int(out[0]), ms=out[1], bytes=out[2], flops=out[3])
+
+
+def cdsl_gemv_noalloc(w, x, y, stream=None):
+    """y[R, N] = x[R, K] w^T through the weight-streaming kernel with its scratch in a fixed
+    array inside the library (no device memory is allocated); see include/cdsl.h."""
+    N, K = w.shape
+    R = x.shape[0]
+    _check(lib().cdsl_gemv_noalloc(w.data_ptr(), N, K, x.data_ptr(), R, y.data_ptr(), stream))
 
 
 def cdsl_last_error(ctx=None) -> str:

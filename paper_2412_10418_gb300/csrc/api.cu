@@ -434,6 +434,8 @@ int validate_all(const cdsl_model_cfg* t, const cdsl_model_cfg* dr, const cdsl_r
 
 }  // namespace
 
+void cdsl::set_thread_error(const char* msg) { g_init_error = msg ? msg : ""; }
+
 extern "C" {
 
 int32_t cdsl_num_weights(const cdsl_model_cfg* cfg) {

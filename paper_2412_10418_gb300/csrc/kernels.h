@@ -73,6 +73,9 @@ constexpr int kPlanSMs = 152;  // GB300: split-K is planned for this many SMs
 GemvPlan plan_gemv(int K, int n_virtual, int n_sm);
 void launch_gemv(const GemmArgs& a, const GemvPlan& p, float* part, int* tile_cnt, cudaStream_t s);
 
+// Message returned by cdsl_last_error(NULL) on this thread.
+void set_thread_error(const char* msg);
+
 // plans and the decision
 void launch_plan_draft(const StepState& st, int j, int tail_slots_per_beam, RowDesc* rows,
                        cudaStream_t s);
