@@ -4,6 +4,8 @@
 
 #include <algorithm>
 #include <array>
+#include <map>
+#include <tuple>
 #include <cstdio>
 #include <cstring>
 #include <string>
@@ -83,6 +85,9 @@ struct cdsl_ctx {
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   std::vector<ProfRec> prof;
+  // TMA descriptors, built on first use: (base, inner, outer, box_outer) -> map
+  std::map<std::tuple<uintptr_t, int, int, int>, CUtensorMap> maps;
+  int map_error = 0;
   std::string err;
 };
 
@@ -94,6 +99,12 @@ int fail(cdsl_ctx* c, int code, const std::string& msg) {
 }
 
 int cuda_check(cdsl_ctx* c, const char* where) {
+  if (c && c->map_error) {
+    const int m = c->map_error;
+    c->map_error = 0;
+    return fail(c, CDSL_ECUDA, std::string(where) + ": cuTensorMapEncodeTiled failed (" +
+                                   std::to_string(m) + ")");
+  }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess)
     return fail(c, CDSL_ECUDA, std::string(where) + ": " + cudaGetErrorString(e));
@@ -209,6 +220,13 @@ size_t carve(cdsl_ctx* c, void* base) {
         const GemvPlan p = plan_gemv(sh[0], sh[1], kPlanSMs);
         part = std::max(part, (size_t)p.splits * 8 * p.tiles * 128);
         tiles = std::max(tiles, (size_t)p.tiles);
+        if (c->dtype == CDSL_DTYPE_BF16 && sh[0] % 64 == 0) {
+          for (int R = 9; R <= std::min(c->R_max, 256); R += 16) {  // every n_pad in use
+            const TcPlan t = plan_tc(sh[0], sh[1], R, kPlanSMs);
+            part = std::max(part, (size_t)t.splits * t.n_pad * t.tiles * 128);
+            tiles = std::max(tiles, (size_t)t.tiles);
+          }
+        }
       }
     }
     c->gemv_part = cv.take<float>(part);
@@ -246,6 +264,8 @@ size_t carve(cdsl_ctx* c, void* base) {
   return (cv.off + 255) & ~size_t(255);
 }
 
+const CUtensorMap& tensor_map(cdsl_ctx* c, const void* base, int inner, int outer, int box_outer);
+
 // Algorithmic bytes of one projection GEMM: every weight once, the activations read once
 // (4 bytes per element: fp32, or bf16 hi + lo), the outputs written once (read-modify-write
 // for the residual add).
@@ -265,7 +285,8 @@ double gemm_bytes(const cdsl_ctx* c, const GemmArgs& a, double* flops) {
 }
 
 void gemm(cdsl_ctx* c, const GemmArgs& a) {
-  const int impl = (c->dtype == CDSL_DTYPE_BF16 && a.R <= 8) ? 1 : 0;
+  const bool bf16 = c->dtype == CDSL_DTYPE_BF16;
+  const int impl = (bf16 && a.R <= 8) ? 1 : (bf16 && tc_supported(a)) ? 2 : 0;
   size_t ev = 0;
   if (c->profiling) {
     while (c->ev_pool.size() < c->ev_used + 2) {
@@ -277,10 +298,22 @@ void gemm(cdsl_ctx* c, const GemmArgs& a) {
     c->ev_used += 2;
     cudaEventRecord(c->ev_pool[ev], c->stream);
   }
-  if (impl == 1)
+  if (impl == 1) {
     launch_gemv(a, plan_gemv(a.K, a.n_virtual, kPlanSMs), c->gemv_part, c->gemv_cnt, c->stream);
-  else
+  } else if (impl == 2) {
+    TcMaps maps;
+    for (int s = 0; s < 3; ++s) {
+      const int seg = s < a.n_seg ? s : 0;
+      maps.w[s] = tensor_map(c, a.w[seg], a.K, a.seg_rows[seg], 64);
+    }
+    const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(a.x);
+    maps.xh = tensor_map(c, xb, a.ldx, c->R_pad, 16);
+    maps.xl = tensor_map(c, xb + a.x_plane, a.ldx, c->R_pad, 16);
+    launch_gemm_tc(maps, a, plan_tc(a.K, a.n_virtual, a.R, kPlanSMs), c->gemv_part, c->gemv_cnt,
+                   c->stream);
+  } else {
     launch_gemm_simt(c->dtype, a, c->stream);
+  }
   if (c->profiling) {
     cudaEventRecord(c->ev_pool[ev + 1], c->stream);
     double fl = 0;
@@ -301,7 +334,19 @@ GemmArgs gemm_base(const cdsl_ctx* c, const ModelW& m, int mode, int K, const vo
   a.R = R;
   a.n_heads = m.cfg.n_heads;
   a.kv = m.kv;
+  a.status = c->st.status;
   return a;
+}
+
+const CUtensorMap& tensor_map(cdsl_ctx* c, const void* base, int inner, int outer, int box_outer) {
+  const auto key = std::make_tuple(reinterpret_cast<uintptr_t>(base), inner, outer, box_outer);
+  auto it = c->maps.find(key);
+  if (it != c->maps.end()) return it->second;
+  CUtensorMap m;
+  std::memset(&m, 0, sizeof m);
+  const int e = encode_bf16_map(&m, base, (uint64_t)inner, (uint64_t)outer, 64, (uint32_t)box_outer);
+  if (e && !c->map_error) c->map_error = e;
+  return c->maps.emplace(key, m).first->second;
 }
 
 // One forward pass of a model over R rows described by `rows`; for lm_rows > 0 the final
@@ -489,6 +534,10 @@ int32_t cdsl_init(const cdsl_model_cfg* target, const void* const* h_target_weig
   }
   carve(c, d_workspace);
   cudaGetLastError();
+  if (c->dtype == CDSL_DTYPE_BF16 && configure_gemm_tc()) {
+    delete c;
+    return fail(nullptr, CDSL_ECUDA, "cannot configure the tensor-core GEMM (shared memory)");
+  }
   cudaMemsetAsync(d_workspace, 0, c->ws_total, c->stream);
   launch_rope_table(c->tgt.rope, c->lrope, target->head_dim, target->rope_theta, c->stream);
   launch_rope_table(c->dft.rope, c->lrope, draft->head_dim, draft->rope_theta, c->stream);

@@ -41,6 +41,7 @@ struct GemmArgs {
   int32_t layer;
   const RowDesc* rows;     // QKV: per-row position and KV destination
   const float2* rope;      // QKV: [pos][hd/2] (cos, sin)
+  int32_t* status;         // device status word (bounded waits report CDSL_ETIMEOUT here)
 };
 
 // Pointer to virtual row v of the segmented weight matrix, nullptr for padding rows.
