@@ -74,6 +74,11 @@ struct cdsl_ctx {
   int32_t* lm_dst = nullptr;
   float* gemv_part = nullptr;   // split-K partial tiles of the weight-streaming GEMM
   int32_t* gemv_cnt = nullptr;  // per-tile arrival counters
+  float* attn_o = nullptr;      // split-KV attention partials (outputs)
+  float* attn_ml = nullptr;     // split-KV attention partials (max, sum)
+  int32_t* attn_cnt = nullptr;  // per-(query block, head) arrival counters
+  int32_t* attn_zmap = nullptr; // prefill: z -> (prompt, query block)
+  int attn_zmax = 0, attn_chunks = 0;
   StepState st{};
   size_t ws_total = 0;
   int phase = PH_NEW;
@@ -232,6 +237,20 @@ size_t carve(cdsl_ctx* c, void* base) {
     c->gemv_part = cv.take<float>(part);
     c->gemv_cnt = cv.take<int32_t>(tiles);
   }
+  {  // split-KV attention scratch
+    const int QB = attn_qblock();
+    const int G = std::max(c->tcfg.n_heads / c->tcfg.n_kv_heads, c->dcfg.n_heads / c->dcfg.n_kv_heads);
+    const int kvh = std::max(c->tcfg.n_kv_heads, c->dcfg.n_kv_heads);
+    const int hd = std::max(c->tcfg.head_dim, c->dcfg.head_dim);
+    auto qbs = [&](int rows) { return (rows * G + QB - 1) / QB; };
+    c->attn_zmax = std::max(std::max(B * qbs(k * (d + 1)), B * qbs(k + 1)), qbs(c->R_p) + B);
+    c->attn_chunks = (c->run.max_prompt + c->run.max_new + attn_chunk() - 1) / attn_chunk();
+    const size_t groups = (size_t)c->attn_zmax * kvh;
+    c->attn_o = cv.take<float>(groups * c->attn_chunks * QB * hd);
+    c->attn_ml = cv.take<float>(groups * c->attn_chunks * QB * 2);
+    c->attn_cnt = cv.take<int32_t>(groups);
+    c->attn_zmap = cv.take<int32_t>((size_t)2 * c->attn_zmax);
+  }
   StepState& s = c->st;
   s.B = B; s.k = k; s.d = d; s.nk = c->nk; s.max_new = c->run.max_new; s.lcap = c->lcap;
   s.reward_head = c->run.reward_head;
@@ -351,12 +370,33 @@ const CUtensorMap& tensor_map(cdsl_ctx* c, const void* base, int inner, int oute
 
 // One forward pass of a model over R rows described by `rows`; for lm_rows > 0 the final
 // norm + LM head run over rows gather[i] (or the first lm_rows rows) into logits.
+// Attention layout of a pass: rows per prompt (dense z mapping) or a host-built z map.
+struct AttnPass {
+  int rows_per_prompt = 0;            // dense: z = b * qb_count + qb
+  const std::vector<int32_t>* zmap = nullptr;  // prefill: (b, qb) pairs for this model
+  int n_chunks = 0;
+};
+
 void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
-             const int32_t* gather, float* logits, float* head_out) {
+             const int32_t* gather, float* logits, float* head_out, const AttnPass& ap) {
   const cdsl_model_cfg& cfg = m.cfg;
   const int D = cfg.d_model, hd = cfg.head_dim, H = cfg.n_heads, KVH = cfg.n_kv_heads;
   const int F = cfg.d_ffn;
   cudaStream_t s = c->stream;
+  AttnArgs at{};
+  at.q = c->qbuf; at.n_heads = H; at.G = H / KVH; at.kv = m.kv; at.rows = rows; at.R = R;
+  at.out = c->X1; at.plane = c->act_plane; at.scale = 1.0f / sqrtf((float)hd);
+  at.n_chunks = ap.n_chunks ? ap.n_chunks : c->attn_chunks;
+  at.part_o = c->attn_o; at.part_ml = c->attn_ml; at.cnt = c->attn_cnt;
+  int n_z;
+  if (ap.zmap) {
+    n_z = (int)ap.zmap->size() / 2;
+    at.zmap = c->attn_zmap;
+    cudaMemcpyAsync(c->attn_zmap, ap.zmap->data(), ap.zmap->size() * 4, cudaMemcpyHostToDevice, s);
+  } else {
+    at.qb_count = (ap.rows_per_prompt * at.G + attn_qblock() - 1) / attn_qblock();
+    n_z = c->B * at.qb_count;
+  }
   launch_embed(c->dtype, rows, R, m.embed, D, c->h, s);
   for (int l = 0; l < cfg.n_layers; ++l) {
     const auto& W = m.layers[l];
@@ -372,8 +412,8 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     q.rows = rows;
     q.rope = m.rope;
     gemm(c, q);
-    launch_attention(c->dtype, c->qbuf, m.kv, l, rows, R, H, c->lcap + c->d + 1, c->X1,
-                     c->act_plane, c->st.status, s);
+    at.layer = l;
+    launch_attn(c->dtype, at, n_z, s);
     GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->X1, H * hd, R);
     o.w[0] = W[W_O]; o.seg_rows[0] = D; o.n_seg = 1; o.n_virtual = D;
     o.out_f32 = c->h; o.ld_out = D;
@@ -405,7 +445,9 @@ void do_lookahead(cdsl_ctx* c) {
   for (int j = 1; j <= c->d; ++j) {
     launch_plan_draft(c->st, j, c->dft.spb, c->rows_d, c->stream);
     const int R = c->B * c->k + (j == 1 ? c->B : 0);
-    forward(c, c->dft, c->rows_d, R, c->B * c->k, nullptr, c->logits, nullptr);
+    AttnPass ap;
+    ap.rows_per_prompt = c->k + (j == 1 ? 1 : 0);
+    forward(c, c->dft, c->rows_d, R, c->B * c->k, nullptr, c->logits, nullptr, ap);
     RowStatsArgs a{};
     a.logits = c->logits; a.R = c->B * c->k; a.V = c->V; a.k = c->k;
     a.x_out = c->st.x; a.logq_out = c->st.logq; a.out_stride = c->d; a.out_off = j - 1;
@@ -416,8 +458,10 @@ void do_lookahead(cdsl_ctx* c) {
 
 void do_verify(cdsl_ctx* c) {
   launch_plan_verify(c->st, c->rows_v, c->stream);
+  AttnPass ap;
+  ap.rows_per_prompt = c->k * (c->d + 1);
   forward(c, c->tgt, c->rows_v, c->R_v, c->R_v, nullptr, c->logits,
-          c->run.reward_head ? c->st.v_head : nullptr);
+          c->run.reward_head ? c->st.v_head : nullptr, ap);
   RowStatsArgs a{};
   a.logits = c->logits; a.R = c->R_v; a.V = c->V; a.k = c->k; a.dp1 = c->d + 1;
   a.next_x = c->st.x; a.amax = c->st.v_amax; a.logp = c->st.v_logp; a.topk = c->st.v_topk;
@@ -534,6 +578,10 @@ int32_t cdsl_init(const cdsl_model_cfg* target, const void* const* h_target_weig
   }
   carve(c, d_workspace);
   cudaGetLastError();
+  if (configure_attention()) {
+    delete c;
+    return fail(nullptr, CDSL_ECUDA, "cannot configure the attention kernel (shared memory)");
+  }
   if (c->dtype == CDSL_DTYPE_BF16 && configure_gemm_tc()) {
     delete c;
     return fail(nullptr, CDSL_ECUDA, "cannot configure the tensor-core GEMM (shared memory)");
@@ -596,14 +644,33 @@ int32_t cdsl_prefill(cdsl_ctx* c, const int32_t* d_prompts, const int32_t* h_pro
       cudaMemcpyAsync(c->lm_gather, gather.data(), 4 * nlm, cudaMemcpyHostToDevice, s);
       cudaMemcpyAsync(c->lm_dst, dst.data(), 4 * nlm, cudaMemcpyHostToDevice, s);
     }
-    forward(c, c->tgt, c->rows_p, R, nlm, c->lm_gather, c->logits, nullptr);
+    // z maps: each prompt present in the chunk, its rows in query blocks
+    std::vector<int> per_prompt(B, 0);
+    int maxpos = 0;
+    for (const RowDesc& rd : rows) { per_prompt[rd.b]++; maxpos = std::max(maxpos, rd.pos); }
+    auto zmap_for = [&](const cdsl_model_cfg& mc) {
+      std::vector<int32_t> z;
+      const int G = mc.n_heads / mc.n_kv_heads;
+      for (int b = 0; b < B; ++b)
+        for (int q = 0; q < (per_prompt[b] * G + attn_qblock() - 1) / attn_qblock(); ++q) {
+          z.push_back(b);
+          z.push_back(q);
+        }
+      return z;
+    };
+    const std::vector<int32_t> zt = zmap_for(c->tcfg), zd = zmap_for(c->dcfg);
+    AttnPass apt, apd;
+    apt.zmap = &zt;
+    apd.zmap = &zd;
+    apt.n_chunks = apd.n_chunks = (maxpos + attn_chunk()) / attn_chunk();
+    forward(c, c->tgt, c->rows_p, R, nlm, c->lm_gather, c->logits, nullptr, apt);
     if (nlm) {
       RowStatsArgs a{};
       a.logits = c->logits; a.R = nlm; a.V = c->V; a.k = c->k;
       a.topk = st.roots; a.dst = c->lm_dst; a.status = st.status;
       launch_row_stats(a, s);
     }
-    forward(c, c->dft, c->rows_p, R, 0, nullptr, nullptr, nullptr);
+    forward(c, c->dft, c->rows_p, R, 0, nullptr, nullptr, nullptr, apd);
     cudaStreamSynchronize(s);  // host row buffers are reused by the next chunk
     rows.clear(); gather.clear(); dst.clear();
   };

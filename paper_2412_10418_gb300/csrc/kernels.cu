@@ -1,5 +1,5 @@
-// kernels.cu -- embedding, RMSNorm (+ reward head), attention over the paged prefix and the
-// beam tails, logits row statistics, row plans, and the CDSL acceptance decision / commit.
+// kernels.cu -- embedding, RMSNorm (+ reward head), logits row statistics, row plans, and the
+// CDSL acceptance decision / commit.
 #include <cuda_bf16.h>
 #include <math.h>
 
@@ -68,66 +68,6 @@ __global__ void k_rmsnorm(const float* h, int D, const T* g, float eps, T* out, 
   if (head_w) {
     hw = block_sum(hw, red);
     if (threadIdx.x == 0) head_out[r] = 1.0f / (1.0f + expf(-hw));
-  }
-}
-
-// ------------------------------------------------------------------------------ attention
-// One block per (row, kv head): the G = n_heads / kvh query heads of that kv head attend to
-// the row's visible keys (prefix [0, n_prefix) through the page table, then its tail slots).
-__device__ __forceinline__ const float* key_row(const KvStore& kv, int layer, const RowDesc& rd,
-                                                int t, int kvsel, int head) {
-  if (t < rd.n_prefix) {
-    const int page = kv.page_table[rd.b * kv.max_pages + (t >> kv.page_shift)];
-    return kv.pool + kv_prefix_offset(kv, layer, page < 0 ? 0 : page, kvsel, head,
-                                      t & ((1 << kv.page_shift) - 1));
-  }
-  return kv.tail + kv_tail_offset(kv, layer, kvsel, rd.tail_base + (t - rd.n_prefix), head);
-}
-
-template <typename T>
-__global__ void k_attention(const float* q, KvStore kv, int layer, const RowDesc* rows,
-                            int n_heads, T* out, size_t plane, float scale) {
-  extern __shared__ float sm[];
-  const int r = blockIdx.x, g = blockIdx.y;
-  const RowDesc rd = rows[r];
-  const int hd = kv.hd, G = n_heads / kv.kvh;
-  const int nkeys = rd.n_prefix + rd.n_tail;
-  float* qs = sm;              // [G][hd]
-  float* sc = sm + G * hd;     // [G][nkeys]
-  __shared__ float inv_sum[16];
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  for (int i = threadIdx.x; i < G * hd; i += blockDim.x)
-    qs[i] = q[(size_t)r * n_heads * hd + (size_t)g * G * hd + i] * scale;
-  __syncthreads();
-  for (int t = wid; t < nkeys; t += nw) {
-    const float* kr = key_row(kv, layer, rd, t, 0, g);
-    for (int gg = 0; gg < G; ++gg) {
-      float s = 0.f;
-      for (int e = lane; e < hd; e += 32) s += qs[gg * hd + e] * kr[e];
-      s = warp_sum(s);
-      if (lane == 0) sc[gg * nkeys + t] = s;
-    }
-  }
-  __syncthreads();
-  for (int gg = wid; gg < G; gg += nw) {
-    float m = -INFINITY;
-    for (int t = lane; t < nkeys; t += 32) m = fmaxf(m, sc[gg * nkeys + t]);
-    m = warp_max(m);
-    float z = 0.f;
-    for (int t = lane; t < nkeys; t += 32) {
-      const float p = expf(sc[gg * nkeys + t] - m);
-      sc[gg * nkeys + t] = p;
-      z += p;
-    }
-    z = warp_sum(z);
-    if (lane == 0) inv_sum[gg] = 1.0f / z;
-  }
-  __syncthreads();
-  for (int i = threadIdx.x; i < G * hd; i += blockDim.x) {
-    const int gg = i / hd, e = i % hd;
-    float acc = 0.f;
-    for (int t = 0; t < nkeys; ++t) acc += sc[gg * nkeys + t] * key_row(kv, layer, rd, t, 1, g)[e];
-    store_act<T>(out, plane, (size_t)r * n_heads * hd + (size_t)g * G * hd + i, acc * inv_sum[gg]);
   }
 }
 
@@ -429,24 +369,6 @@ void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, f
                     float* head_out, cudaStream_t s) {
   DISPATCH(dtype, k_rmsnorm<T><<<R, 256, 0, s>>>(h, D, (const T*)gain, eps, (T*)out, plane,
                                                  gather, head_w, head_out));
-}
-
-void launch_attention(int dtype, const float* q, KvStore kv, int layer, const RowDesc* rows,
-                      int R, int n_heads, int max_keys, void* out, size_t plane,
-                      int32_t* status, cudaStream_t s) {
-  const int G = n_heads / kv.kvh;
-  const size_t smem = sizeof(float) * ((size_t)G * kv.hd + (size_t)G * max_keys);
-  const float scale = 1.0f / sqrtf((float)kv.hd);
-  dim3 grid(R, kv.kvh);
-  DISPATCH(dtype, {
-    static int configured = 0;
-    if (smem > 48 * 1024 && configured < (int)smem) {
-      cudaFuncSetAttribute(k_attention<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      configured = (int)smem;
-    }
-    k_attention<T><<<grid, 128, smem, s>>>(q, kv, layer, rows, n_heads, (T*)out, plane, scale);
-  });
-  (void)status;
 }
 
 void launch_row_stats(const RowStatsArgs& a, cudaStream_t s) {

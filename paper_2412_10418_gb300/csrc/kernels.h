@@ -45,9 +45,24 @@ void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int 
 void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
                     void* out, size_t plane, const int32_t* gather, const float* head_w,
                     float* head_out, cudaStream_t s);
-void launch_attention(int dtype, const float* q, KvStore kv, int layer, const RowDesc* rows,
-                      int R, int n_heads, int max_keys, void* out, size_t plane,
-                      int32_t* status, cudaStream_t s);
+// Attention of a pass (attention.cu). Blocks: (prefix chunk of attn_chunk() positions, kv
+// head, z) with z -> (prompt, query block of attn_qblock() query vectors) either dense
+// (b = z / qb_count) or from zmap[2z], zmap[2z+1]. Scratch: part_o
+// [n_z][kvh][n_chunks][qblock][hd], part_ml [n_z][kvh][n_chunks][qblock][2], cnt [n_z][kvh]
+// (zero between launches).
+struct AttnArgs {
+  const float* q; int32_t n_heads, G;
+  KvStore kv; int32_t layer;
+  const RowDesc* rows; int32_t R;
+  void* out; size_t plane; float scale;
+  int32_t n_chunks, qb_count;
+  const int32_t* zmap;
+  float* part_o; float* part_ml; int32_t* cnt;
+};
+int attn_chunk();
+int attn_qblock();
+int configure_attention();
+void launch_attn(int dtype, const AttnArgs& a, int n_z, cudaStream_t s);
 // Row statistics of logits rows: argmax (lower id on ties), log-sum-exp, top-k, log p.
 //   draft mode  (dp1 == 0): x[r*out_stride + out_off] = argmax, logq[...] = log q(argmax)
 //   verify mode (dp1 == d+1): amax[r], topk[r, k], logp of the next drafted token
