@@ -228,7 +228,7 @@ size_t carve(cdsl_ctx* c, void* base) {
         if (c->dtype == CDSL_DTYPE_BF16 && sh[0] % 64 == 0) {
           for (int R = 9; R <= std::min(c->R_max, 256); R += 16) {  // every n_pad in use
             const TcPlan t = plan_tc(sh[0], sh[1], R, kPlanSMs);
-            part = std::max(part, (size_t)t.splits * t.n_pad * t.tiles * 128);
+            part = std::max(part, tc_scratch_floats(t));
             tiles = std::max(tiles, (size_t)t.tiles);
           }
         }
@@ -304,8 +304,11 @@ double gemm_bytes(const cdsl_ctx* c, const GemmArgs& a, double* flops) {
 }
 
 void gemm(cdsl_ctx* c, const GemmArgs& a) {
+  // bf16: the tensor-core kernel for every shape it supports (it streams weights faster than
+  // the CUDA-core GEMV even at 4-8 rows); the weight-streaming GEMV otherwise at <= 8 rows;
+  // float32 (and anything else): the CUDA-core tiled GEMM.
   const bool bf16 = c->dtype == CDSL_DTYPE_BF16;
-  const int impl = (bf16 && a.R <= 8) ? 1 : (bf16 && tc_supported(a)) ? 2 : 0;
+  const int impl = (bf16 && tc_supported(a)) ? 2 : (bf16 && a.R <= 8) ? 1 : 0;
   size_t ev = 0;
   if (c->profiling) {
     while (c->ev_pool.size() < c->ev_used + 2) {

@@ -64,13 +64,18 @@ __device__ __forceinline__ const T* virtual_row(const GemmArgs& a, int v) {
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }
 
 // Apply the epilogue to a finished fp32 tile: tile[r * ldt + v] holds y for activation row
-// r0 + r and virtual row v0 + v (v in [0, 128)), for r in [0, rt). Called by all threads of
-// a block; the caller synchronizes before and after.
+// r0 + r and virtual row v0 + v (v in [0, 128)), for r in [0, rt). Run by `nthr` threads
+// (tid = 0 .. nthr-1; all threads of the block by default); the caller synchronizes them
+// before and after.
 template <typename T>
 __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const float* tile,
-                              int ldt) {
+                              int ldt, int tid = -1, int nthr = -1) {
+  if (tid < 0) {
+    tid = threadIdx.x;
+    nthr = blockDim.x;
+  }
   const int n_items = rt * 128;
-  for (int idx = threadIdx.x; idx < n_items; idx += blockDim.x) {
+  for (int idx = tid; idx < n_items; idx += nthr) {
     const int r = idx >> 7, v = idx & 127;
     const int row = r0 + r;
     if (row >= a.R) continue;

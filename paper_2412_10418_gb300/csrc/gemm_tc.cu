@@ -4,16 +4,24 @@
 // two 64-row TMA boxes so that a tile may draw its halves from different segments: gate/up
 // interleave, q/k/v boundaries) and the activation rows are the N operand (N = R rounded up
 // to 16, 16..256). Both operands are K-major bf16 in 128-byte-swizzled shared-memory tiles;
-// the accumulator lives in TMEM (fp32, N columns). The activations come as the hi and lo bf16
-// planes of the split, so each 16-deep K step issues two MMAs into the same accumulator.
+// the accumulator lives in TMEM (fp32). The activations come as the hi and lo bf16 planes of
+// the split, so each 16-deep K step issues two MMAs into the same accumulator.
 //
-// Block = 4 warps: lane 0 of warp 0 issues TMA loads through a ring of mbarrier-guarded
-// stages, lane 0 of warp 1 issues the MMAs and releases each stage with tcgen05.commit; then
-// all four warps read their 32 TMEM lanes each. K is split across blocks when the tile count
-// alone cannot fill the GPU; as in the weight-streaming kernel, partial tiles go to scratch
-// and the last block of a tile sums them in split order and runs the fused epilogue.
-// Every wait is bounded in time; on expiry the block latches CDSL_ETIMEOUT, waits (bounded)
-// for its own copies in flight, frees its TMEM and returns.
+// Persistent stream-K schedule: a fixed grid of blocks (two per SM when the ring fits in half
+// the shared memory) divides the tiles x 64-wide K blocks evenly, so there is no partial last
+// wave. A block walks its contiguous range of (tile, k-block) units; a run of units within one
+// tile is a segment. Warp 0 (one lane) streams weights and activations with TMA through a
+// ring of mbarrier-guarded stages; warp 1 (one lane) issues the MMAs into one of two TMEM
+// accumulators and commits; warps 2-5 drain a finished accumulator (TMEM -> registers ->
+// shared memory) while the next segment accumulates into the other one. A segment covering a
+// whole tile runs the fused epilogue directly; otherwise its partial tile goes to scratch and
+// the last contributing block of that tile adds the partials in block order (a deterministic
+// sum) and runs the epilogue.
+//
+// Programmatic dependent launch: weights do not depend on the previous kernel, so the TMA
+// lane issues the first ring's weight loads before griddepcontrol.wait and the activation
+// loads after it; every other dependent access comes after the wait. Every wait on an mbarrier
+// is bounded in time; on expiry the block latches CDSL_ETIMEOUT and winds down.
 #include <cudaTypedefs.h>
 
 #include <algorithm>
@@ -26,12 +34,12 @@ namespace cdsl {
 namespace {
 
 constexpr int kMaxStages = 8;
-constexpr int kStageBudget = 220 * 1024;            // ring memory a plan may use
-constexpr int kMaxDynSmem = kStageBudget + 1024;    // + alignment slack (static smem is extra)
-constexpr int kTileLd = 132;   // fp32 epilogue tile row pitch (128 + 4 against bank conflicts)
-constexpr int kThreads = 128;
+constexpr int kTileLd = 132;     // fp32 epilogue tile row pitch (128 + 4 against bank conflicts)
+constexpr int kEpRowsMax = 64;   // activation rows drained per epilogue chunk (at most)
+constexpr int kThreads = 192;    // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kEpThreads = 128;
 
-__device__ __forceinline__ uint32_t tmem_cols(int n_pad) {
+__host__ __device__ __forceinline__ uint32_t tmem_cols_for(int n_pad) {
   uint32_t c = 32;
   while (c < (uint32_t)n_pad) c <<= 1;
   return c;
@@ -55,142 +63,268 @@ __device__ __forceinline__ void half_source(const GemmArgs& a, int vstart, int* 
   }
 }
 
+// Stream-K partition: block c owns units [start(c), start(c + 1)) (U * C < 2^31, checked on
+// the host).
+__device__ __forceinline__ int unit_start(int c, int U, int C) { return c * U / C; }
+__device__ __forceinline__ int unit_owner(int u, int U, int C) { return ((u + 1) * C - 1) / U; }
+
+constexpr int kMaxContrib = 256;   // contributors to one tile (bounded on the host)
+constexpr int kMaxSplit = 4;       // target blocks per tile when tiles are few
+
 __global__ void __launch_bounds__(kThreads, 1)
     k_gemm_tc(const __grid_constant__ TcMaps maps, const __grid_constant__ GemmArgs a, TcPlan p,
               float* part, int* tile_cnt) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
-  __shared__ __align__(8) uint64_t done_bar;
+  __shared__ __align__(8) uint64_t accf_bar[2];
+  __shared__ __align__(8) uint64_t acce_bar[2];
   __shared__ uint32_t tmem_base;
   __shared__ int s_abort, s_last;
+  __shared__ int s_slot_off[kMaxContrib];   // reducer: scratch offset (floats) per contributor
 
   uint8_t* smem = smem_raw + ((1024 - (tc::smem_u32(smem_raw) & 1023)) & 1023);
-  const int tile = blockIdx.x, split = blockIdx.y;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int v0 = tile * 128;
-  const int total_kb = a.K >> 6;
-  const int kb0 = split * p.kb_per_split;
-  const int nkb = min(p.kb_per_split, total_kb - kb0);
-  const int S = p.stages, NP = p.n_pad;
+  const int NP = p.n_pad, S = p.stages, KBT = p.kb_total;
   const uint32_t stage_bytes = 16384u + 256u * NP;
-  const uint32_t ncols = tmem_cols(NP);
+  const int kEpRows = p.ep_rows;
+  float* tileS = reinterpret_cast<float*>(smem + (size_t)S * stage_bytes);  // [ep_rows][kTileLd]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x, C = gridDim.x;
+  const int U = p.tiles * KBT;
+  const int u0 = unit_start(c, U, C), u1 = unit_start(c + 1, U, C);
+  // hi and lo rows are contiguous in each stage: one MMA with N = 2*NP covers both (the
+  // accumulator then holds W.hi in columns [0, NP) and W.lo in [NP, 2NP)); above N = 256 they
+  // are two MMAs into one accumulator.
+  const bool fused = 2 * NP <= 256;
+  const uint32_t acc_cols = tmem_cols_for(fused ? 2 * NP : NP);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       tc::mbar_init(&full_bar[s], 1);
       tc::mbar_init(&empty_bar[s], 1);
     }
-    tc::mbar_init(&done_bar, 1);
+    for (int i = 0; i < 2; ++i) {
+      tc::mbar_init(&accf_bar[i], 1);
+      tc::mbar_init(&acce_bar[i], kEpThreads);
+    }
     s_abort = 0;
     tc::fence_mbar_init();
   }
-  if (warp == 1) tc::tmem_alloc(&tmem_base, ncols);
+  if (warp == 1) tc::tmem_alloc(&tmem_base, 2 * acc_cols);
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
+  if (threadIdx.x == 0) pdl_launch_dependents();
   const uint32_t tmem = tmem_base;
 
-  if (warp == 0 && lane == 0) {
-    // ---------------- TMA producer
-    int m0, y0, m1, y1;
-    half_source(a, v0, &m0, &y0);
-    half_source(a, v0 + 64, &m1, &y1);
-    const uint64_t pol = tc::policy_evict_first();
-    int issued = 0;
-    bool aborted = false;
-    for (int i = 0; i < nkb; ++i) {
-      const int s = i % S, use = i / S;
-      if (use > 0 && !tc::mbar_wait(&empty_bar[s], (use - 1) & 1, a.status)) {
-        aborted = true;
-        break;
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer
+      const uint64_t pol = tc::policy_evict_first();
+      const int n = (int)(u1 - u0);
+      const int pre = min(S, n);
+      bool aborted = false;
+      int issued = 0;
+      int t_cur = u0 / KBT, kb_cur = u0 % KBT;   // unit u0 + i, advanced incrementally
+      auto load_w = [&](int i, int t, int kb) {
+        int m0, y0, m1, y1;
+        half_source(a, t * 128, &m0, &y0);
+        half_source(a, t * 128 + 64, &m1, &y1);
+        uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
+        tc::tma_load_2d_hint(st, &maps.w[m0], kb * 64, y0, &full_bar[i % S], pol);
+        tc::tma_load_2d_hint(st + 8192, &maps.w[m1], kb * 64, y1, &full_bar[i % S], pol);
+      };
+      auto load_x = [&](int i, int kb) {
+        uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
+        for (int j = 0; j < NP / 16; ++j) {
+          tc::tma_load_2d(st + 16384 + j * 2048, &maps.xh, kb * 64, j * 16, &full_bar[i % S]);
+          tc::tma_load_2d(st + 16384 + NP * 128 + j * 2048, &maps.xl, kb * 64, j * 16,
+                          &full_bar[i % S]);
+        }
+      };
+      // the first ring's weights do not depend on the previous kernel
+      for (int i = 0; i < pre; ++i) {
+        tc::mbar_expect_tx(&full_bar[i], stage_bytes);
+        load_w(i, t_cur, kb_cur);
+        if (++kb_cur == KBT) { kb_cur = 0; ++t_cur; }
       }
-      uint8_t* st = smem + (size_t)s * stage_bytes;
-      tc::mbar_expect_tx(&full_bar[s], stage_bytes);
-      const int x = (kb0 + i) * 64;
-      tc::tma_load_2d_hint(st, &maps.w[m0], x, y0, &full_bar[s], pol);
-      tc::tma_load_2d_hint(st + 8192, &maps.w[m1], x, y1, &full_bar[s], pol);
-      for (int j = 0; j < NP / 16; ++j) {
-        tc::tma_load_2d(st + 16384 + j * 2048, &maps.xh, x, j * 16, &full_bar[s]);
-        tc::tma_load_2d(st + 16384 + NP * 128 + j * 2048, &maps.xl, x, j * 16, &full_bar[s]);
+      pdl_wait();
+      {
+        int kb = u0 % KBT;
+        for (int i = 0; i < pre; ++i) {
+          load_x(i, kb);
+          if (++kb == KBT) kb = 0;
+        }
       }
-      ++issued;
+      issued = pre;
+      for (int i = pre; i < n; ++i) {
+        const int s = i % S, use = i / S;
+        if (!tc::mbar_wait(&empty_bar[s], (use - 1) & 1, a.status)) {
+          aborted = true;
+          break;
+        }
+        tc::mbar_expect_tx(&full_bar[s], stage_bytes);
+        load_w(i, t_cur, kb_cur);
+        load_x(i, kb_cur);
+        if (++kb_cur == KBT) { kb_cur = 0; ++t_cur; }
+        ++issued;
+      }
+      if (aborted) {
+        s_abort = 1;
+        for (int i = max(0, issued - S); i < issued; ++i)
+          tc::mbar_wait(&full_bar[i % S], (i / S) & 1, a.status);
+      }
     }
-    if (aborted) {
-      s_abort = 1;
-      // let the copies already in flight land before the block can exit
-      for (int i = max(0, issued - S); i < issued; ++i)
-        tc::mbar_wait(&full_bar[i % S], (i / S) & 1, a.status);
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer
+      const uint32_t idesc = tc::idesc_bf16_f32(128, fused ? 2 * NP : NP);
+      int seg = 0;
+      int u = u0;
+      bool ok = true;
+      while (u < u1 && ok) {
+        const int seg_end = min(u1, (u / KBT + 1) * KBT);
+        const int acc = seg & 1;
+        if (seg >= 2 && !tc::mbar_wait(&acce_bar[acc], ((seg >> 1) - 1) & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        tc::tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)acc * acc_cols;
+        const int seg_begin = u;
+        for (; u < seg_end; ++u) {
+          const int i = (int)(u - u0), s = i % S, use = i / S;
+          if (!tc::mbar_wait(&full_bar[s], use & 1, a.status)) {
+            ok = false;
+            break;
+          }
+          tc::tc_fence_after();
+          const uint32_t sa = tc::smem_u32(smem + (size_t)s * stage_bytes);
+          const uint64_t da = tc::desc_sw128(sa);
+          const uint64_t dh = tc::desc_sw128(sa + 16384);
+          const uint64_t dl = tc::desc_sw128(sa + 16384 + NP * 128);
+          const bool first = (u == seg_begin);
+          if (fused) {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk)   // 4 x K=16 per stage; +32 bytes = +2 in the desc
+              tc::umma_bf16(d, da + 2 * kk, dh + 2 * kk, idesc, (first && kk == 0) ? 0u : 1u);
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < 4; ++kk) {
+              tc::umma_bf16(d, da + 2 * kk, dh + 2 * kk, idesc, (first && kk == 0) ? 0u : 1u);
+              tc::umma_bf16(d, da + 2 * kk, dl + 2 * kk, idesc, 1u);
+            }
+          }
+          tc::umma_commit(&empty_bar[s]);
+        }
+        tc::umma_commit(&accf_bar[acc]);
+        ++seg;
+      }
+      if (!ok) s_abort = 1;
     }
-  } else if (warp == 1 && lane == 0) {
-    // ---------------- MMA issuer
-    const uint32_t idesc = tc::idesc_bf16_f32(128, NP);
-    for (int i = 0; i < nkb; ++i) {
-      const int s = i % S, use = i / S;
-      if (!tc::mbar_wait(&full_bar[s], use & 1, a.status)) {
+  } else {
+    // ---------------- epilogue warps 2..5: TMEM lanes 32*(warp % 4) .. +31
+    const int etid = threadIdx.x - 64;
+    const int quarter = warp & 3;
+    pdl_wait();
+    int seg = 0;
+    int u = u0;
+    const int R = min(a.R, NP);
+    while (u < u1) {
+      const int t = u / KBT;
+      const int seg_end = min(u1, (t + 1) * KBT);
+      const bool whole = (u % KBT) == 0 && seg_end == (t + 1) * KBT;
+      const int acc = seg & 1;
+      if (!tc::mbar_wait(&accf_bar[acc], (seg >> 1) & 1, a.status)) {
         s_abort = 1;
         break;
       }
       tc::tc_fence_after();
-      const uint32_t sa = tc::smem_u32(smem + (size_t)s * stage_bytes);
-      const uint64_t da = tc::desc_sw128(sa);
-      const uint64_t dh = tc::desc_sw128(sa + 16384);
-      const uint64_t dl = tc::desc_sw128(sa + 16384 + NP * 128);
+      const uint32_t d = tmem + (uint32_t)acc * acc_cols + ((uint32_t)(quarter * 32) << 16);
+      const int slot = (t == u0 / KBT) ? 0 : 1;
+      float* my_part = part + ((size_t)(c * 2 + slot) * NP) * 128;
+      for (int r0 = 0; r0 < NP; r0 += kEpRows) {
+        const int rows = min(kEpRows, NP - r0);
+        for (int c0 = 0; c0 < rows; c0 += 16) {
+          float v[16];
+          tc::tmem_ld16(d + (uint32_t)(r0 + c0), v);
+          if (fused) {
+            float w[16];
+            tc::tmem_ld16(d + (uint32_t)(NP + r0 + c0), w);
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {   // 4 x K=16 per 64-wide stage; +32 bytes = +2 in the desc
-        tc::umma_bf16(tmem, da + 2 * kk, dh + 2 * kk, idesc, (i | kk) != 0);
-        tc::umma_bf16(tmem, da + 2 * kk, dl + 2 * kk, idesc, 1);
+            for (int i = 0; i < 16; ++i) v[i] += w[i];
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) tileS[(c0 + i) * kTileLd + quarter * 32 + lane] = v[i];
+        }
+        tc::named_barrier(1, kEpThreads);
+        const int rt = max(0, min(rows, R - r0));
+        if (whole) {
+          tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, etid, kEpThreads);
+        } else {
+          for (int i = etid; i < rt * 128; i += kEpThreads) {
+            const int r = i >> 7, v = i & 127;
+            my_part[(size_t)(r0 + r) * 128 + v] = tileS[r * kTileLd + v];
+          }
+        }
+        tc::named_barrier(1, kEpThreads);
       }
-      tc::umma_commit(&empty_bar[s]);
-    }
-    tc::umma_commit(&done_bar);
-  }
-  __syncwarp();
-  const bool ok = tc::mbar_wait(&done_bar, 0, a.status);
-  tc::tc_fence_after();
-  __syncthreads();
-
-  float* tileS = reinterpret_cast<float*>(smem);   // [NP][kTileLd], reuses the drained stages
-  const bool good = ok && !s_abort;
-  if (good) {
-    for (int c0 = 0; c0 < NP; c0 += 16) {
-      float v[16];
-      tc::tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+      tc::tc_fence_before();
+      tc::mbar_arrive(&acce_bar[acc]);   // accumulator drained: the MMA lane may reuse it
+      if (!whole) {
+        const int cf = unit_owner(t * KBT, U, C);
+        const int cl = unit_owner((t + 1) * KBT - 1, U, C);
+        __threadfence();
+        tc::named_barrier(1, kEpThreads);
+        if (etid == 0) s_last = (atomicAdd(tile_cnt + t, 1) == cl - cf);
+        tc::named_barrier(1, kEpThreads);
+        if (s_last) {
+          __threadfence();
+          // scratch slot of every contributor: its first segment -> 0, its last -> 1
+          for (int j = etid; j <= cl - cf; j += kEpThreads) {
+            const int cc = cf + j;
+            const int sl = (t == unit_start(cc, U, C) / KBT) ? 0 : 1;
+            s_slot_off[j] = (cc * 2 + sl) * NP * 128;
+          }
+          tc::named_barrier(1, kEpThreads);
+          const int ncontrib = cl - cf + 1;
+          for (int r0 = 0; r0 < R; r0 += kEpRows) {
+            const int rt = min(kEpRows, R - r0);
+            // float4 groups: 32 per activation row; all contributors' loads in flight together
+            for (int i = etid; i < rt * 32; i += kEpThreads) {
+              const int off = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
+              float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+              int j = 0;
+              for (; j + 4 <= ncontrib; j += 4) {
+                float4 v[4];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) tileS[(c0 + i) * kTileLd + warp * 32 + lane] = v[i];
+                for (int q = 0; q < 4; ++q)
+                  v[q] = __ldcg(reinterpret_cast<const float4*>(part + s_slot_off[j + q] + off));
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                  sum.x += v[q].x; sum.y += v[q].y; sum.z += v[q].z; sum.w += v[q].w;
+                }
+              }
+              for (; j < ncontrib; ++j) {
+                const float4 v = __ldcg(reinterpret_cast<const float4*>(part + s_slot_off[j] + off));
+                sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
+              }
+              *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
+            }
+            tc::named_barrier(1, kEpThreads);
+            tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, etid, kEpThreads);
+            tc::named_barrier(1, kEpThreads);
+          }
+          if (etid == 0) tile_cnt[t] = 0;
+        }
+      }
+      u = seg_end;
+      ++seg;
     }
   }
   tc::tc_fence_before();
   __syncthreads();
-  if (warp == 1) tc::tmem_dealloc(tmem, ncols);
-  if (!good) return;
-
-  const int R = min(a.R, NP);
-  if (p.splits == 1) {
-    tile_epilogue<__nv_bfloat16>(a, v0, 0, R, tileS, kTileLd);
-    return;
-  }
-  const int tiles = gridDim.x;
-  for (int i = threadIdx.x; i < R * 128; i += kThreads) {
-    const int r = i >> 7, v = i & 127;
-    part[((size_t)(split * NP + r) * tiles + tile) * 128 + v] = tileS[r * kTileLd + v];
-  }
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(tile_cnt + tile, 1) == p.splits - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  for (int i = threadIdx.x; i < R * 128; i += kThreads) {
-    const int r = i >> 7, v = i & 127;
-    float s = 0.f;
-    for (int sp = 0; sp < p.splits; ++sp)
-      s += __ldcg(part + ((size_t)(sp * NP + r) * tiles + tile) * 128 + v);
-    tileS[r * kTileLd + v] = s;
-  }
-  __syncthreads();
-  tile_epilogue<__nv_bfloat16>(a, v0, 0, R, tileS, kTileLd);
-  if (threadIdx.x == 0) tile_cnt[tile] = 0;
+  if (warp == 1) tc::tmem_dealloc(tmem, 2 * acc_cols);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -199,27 +333,48 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 bool tc_supported(const GemmArgs& a) {
   if (a.K % 64 || a.R < 1 || a.R > 256) return false;
+  // 32-bit stream-K unit arithmetic and at most kMaxContrib blocks per tile
+  const long long units = (long long)((a.n_virtual + 127) / 128) * (a.K / 64);
+  if (a.K / 64 >= kMaxContrib || units * 4 * kPlanSMs >= (1LL << 31)) return false;
   for (int s = 0; s + 1 < a.n_seg; ++s)
     if (a.mode != EPI_SWIGLU && a.seg_rows[s] % 64) return false;
   return true;
 }
 
-TcPlan plan_tc(int K, int n_virtual, int R, int n_sm) {
+TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm) {
   TcPlan p{};
   p.n_pad = (R + 15) / 16 * 16;
   p.tiles = (n_virtual + 127) / 128;
-  const int total_kb = K / 64;
+  p.kb_total = K / 64;
   const size_t stage = 16384 + 256 * (size_t)p.n_pad;
-  const int per_sm = (4 * stage + 2048 <= 113 * 1024) ? 2 : 1;
-  p.stages = per_sm == 2 ? 4 : (int)std::max<size_t>(2, std::min<size_t>(kMaxStages, kStageBudget / stage));
-  const int target = per_sm * n_sm;
-  int splits = std::max(1, (target + p.tiles / 2) / p.tiles);
-  splits = std::min(splits, total_kb);
-  p.kb_per_split = (total_kb + splits - 1) / splits;
-  p.splits = (total_kb + p.kb_per_split - 1) / p.kb_per_split;
-  p.smem = std::max((size_t)p.stages * stage, (size_t)p.n_pad * kTileLd * 4) + 1024;
+  // two blocks per SM when three stages fit in half the shared memory, else one; the
+  // epilogue drains 16 activation rows at a time when that frees room for another stage
+  const size_t half = 113 * 1024;
+  auto fit = [&](size_t budget, int ep) {
+    return (int)std::min<size_t>(kMaxStages, (budget - (size_t)ep * kTileLd * 4 - 1024) / stage);
+  };
+  int per_sm = 1;
+  size_t budget = 220 * 1024;
+  const int ep_big = std::min(p.n_pad, kEpRowsMax);
+  if (force_per_sm >= 3) {   // more, shallower blocks (measurement aid)
+    per_sm = force_per_sm;
+    budget = (227 * 1024) / force_per_sm - 1024;
+  } else if ((force_per_sm == 2 || force_per_sm == 0) && fit(half, 16) >= 3) {
+    per_sm = 2;
+    budget = half;
+  }
+  p.ep_rows = fit(budget, 16) > fit(budget, ep_big) ? 16 : ep_big;
+  p.stages = fit(budget, p.ep_rows);
+  const size_t tile = (size_t)p.ep_rows * kTileLd * 4;
+  // at most kMaxSplit blocks share a tile: the fixup then stays cheap next to the streaming
+  const long long units = (long long)p.tiles * p.kb_total;
+  p.ctas = (int)std::min<long long>(std::min<long long>(units, (long long)per_sm * n_sm),
+                                    (long long)p.tiles * kMaxSplit);
+  p.smem = (size_t)p.stages * stage + tile + 1024;
   return p;
 }
+
+size_t tc_scratch_floats(const TcPlan& p) { return (size_t)p.ctas * 2 * p.n_pad * 128; }
 
 int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                     uint32_t box_inner, uint32_t box_outer) {
@@ -244,16 +399,25 @@ int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
 }
 
 int configure_gemm_tc() {
-  return cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxDynSmem) ==
-                 cudaSuccess
+  return cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              220 * 1024 + 1024) == cudaSuccess
              ? 0
              : -1;
 }
 
 void launch_gemm_tc(const TcMaps& maps, const GemmArgs& a, const TcPlan& p, float* part,
                     int* tile_cnt, cudaStream_t s) {
-  dim3 grid(p.tiles, p.splits);
-  k_gemm_tc<<<grid, kThreads, p.smem, s>>>(maps, a, p, part, tile_cnt);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.ctas);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = p.smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, k_gemm_tc, maps, a, p, part, tile_cnt);
 }
 
 }  // namespace cdsl

@@ -89,14 +89,16 @@ constexpr int kPlanSMs = 152;  // GB300: split-K is planned for this many SMs
 GemvPlan plan_gemv(int K, int n_virtual, int n_sm);
 void launch_gemv(const GemmArgs& a, const GemvPlan& p, float* part, int* tile_cnt, cudaStream_t s);
 
-// Tensor-core GEMM (tcgen05, TMEM, TMA) for bf16 weights and 1..256 activation rows.
-// maps: TMA descriptors of the weight segments (128-byte swizzle, 64x64 boxes) and of the
-// hi / lo activation planes (64x16 boxes). Scratch as for the weight-streaming GEMM:
-// part [splits][n_pad][tiles][128] floats, one arrival counter per tile.
+// Tensor-core GEMM (tcgen05, TMEM, TMA) for bf16 weights and 1..256 activation rows, on a
+// persistent stream-K grid of `ctas` blocks. maps: TMA descriptors of the weight segments
+// (128-byte swizzle, 64x64 boxes) and of the hi / lo activation planes (64x16 boxes).
+// Scratch: part [ctas][2][n_pad][128] floats (tc_scratch_floats), one arrival counter per
+// tile (zero between launches). Launched with programmatic dependent launch allowed.
 struct TcMaps { CUtensorMap w[3]; CUtensorMap xh, xl; };
-struct TcPlan { int tiles, splits, kb_per_split, n_pad, stages; size_t smem; };
+struct TcPlan { int tiles, kb_total, ctas, n_pad, stages, ep_rows; size_t smem; };
 bool tc_supported(const GemmArgs& a);
-TcPlan plan_tc(int K, int n_virtual, int R, int n_sm);
+TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm = 0);
+size_t tc_scratch_floats(const TcPlan& p);
 int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                     uint32_t box_inner, uint32_t box_outer);
 int configure_gemm_tc();
