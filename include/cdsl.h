@@ -168,10 +168,12 @@ CDSL_API int32_t cdsl_get_tokens(cdsl_ctx* ctx, int32_t* d_tokens, int32_t* d_le
 CDSL_API int32_t cdsl_get_counters(cdsl_ctx* ctx, int64_t* h_counters);
 
 /* Kernel timing (a measurement aid; the paper has no counterpart). With enable != 0 every
- * projection-GEMM launch of the following calls is bracketed by CUDA events on the context's
- * stream and cdsl_step launches its kernels directly instead of through its graph.
- * cdsl_get_profile synchronizes the stream and returns, for GEMM implementation `impl`
- * (0 = CUDA-core tiled GEMM, 1 = weight-streaming GEMV, 2 = tcgen05 tensor-core GEMM),
+ * kernel launch of the following calls is bracketed by CUDA events on the context's stream
+ * and cdsl_step launches its kernels directly instead of through its graph.
+ * cdsl_get_profile synchronizes the stream and returns, for kernel class `impl`
+ * (0 = CUDA-core tiled GEMM, 1 = weight-streaming GEMV, 2 = tcgen05 tensor-core GEMM,
+ * 3 = attention, 4 = RMSNorm, 5 = logits row statistics, 6 = embedding, 7 = plans, decision
+ * and commit; bytes and flops are filled in for the GEMM classes only),
  * h_out[4] = {launches, total milliseconds, algorithmic bytes (weights read once, activations
  * read, outputs written), flops} over the launches recorded since cdsl_profile last enabled
  * or disabled timing (each call of cdsl_profile clears the record). */

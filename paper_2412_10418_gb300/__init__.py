@@ -185,6 +185,8 @@ def cdsl_profile(ctx, enable: bool):
 
 
 GEMM_IMPLS = {0: "gemm_simt", 1: "gemv_stream", 2: "gemm_tc"}
+KERNEL_CLASSES = {0: "gemm_simt", 1: "gemv_stream", 2: "gemm_tc", 3: "attention", 4: "rmsnorm",
+                  5: "row_stats", 6: "embed", 7: "step_logic"}
 
 
 def cdsl_get_profile(ctx, impl: int):

@@ -144,7 +144,8 @@ int check_run(const cdsl_run_cfg* r, int vocab, std::string* why) {
   if (r->k < 1 || r->k > 16 || r->k > vocab) return bad("k must be in 1..16");
   if (r->d < 1 || r->d > 16) return bad("d must be in 1..16");
   if (r->max_prompt < 1 || r->max_new < 1) return bad("max_prompt and max_new must be >= 1");
-  if ((long long)r->max_prompt + r->max_new > (1 << 20)) return bad("sequence too long");
+  if ((long long)r->max_prompt + r->max_new > (long long)attn_max_chunks() * attn_chunk())
+    return bad("max_prompt + max_new exceeds the attention limit (4032 positions)");
   if (r->n_keywords < 1 || r->n_keywords > 32) return bad("n_keywords must be in 1..32");
   const int ps = r->page_size ? r->page_size : 64;
   if (ps < 16 || ps > 256 || (ps & (ps - 1))) return bad("page_size must be a power of two in 16..256");
@@ -246,8 +247,9 @@ size_t carve(cdsl_ctx* c, void* base) {
     c->attn_zmax = std::max(std::max(B * qbs(k * (d + 1)), B * qbs(k + 1)), qbs(c->R_p) + B);
     c->attn_chunks = (c->run.max_prompt + c->run.max_new + attn_chunk() - 1) / attn_chunk();
     const size_t groups = (size_t)c->attn_zmax * kvh;
-    c->attn_o = cv.take<float>(groups * c->attn_chunks * QB * hd);
-    c->attn_ml = cv.take<float>(groups * c->attn_chunks * QB * 2);
+    const size_t parts = (size_t)c->attn_chunks + 1;   // prefix chunks + the tail chunk
+    c->attn_o = cv.take<float>(groups * parts * QB * hd);
+    c->attn_ml = cv.take<float>(groups * parts * QB * 2);
     c->attn_cnt = cv.take<int32_t>(groups);
     c->attn_zmap = cv.take<int32_t>((size_t)2 * c->attn_zmax);
   }
@@ -303,26 +305,42 @@ double gemm_bytes(const cdsl_ctx* c, const GemmArgs& a, double* flops) {
   return rows * a.K * wsz + 4.0 * a.R * a.K + out;
 }
 
+// Kernel timing (cdsl_profile): bracket one launch of class `cls` with CUDA events.
+enum { K_GEMM_SIMT = 0, K_GEMV = 1, K_GEMM_TC = 2, K_ATTN = 3, K_NORM = 4, K_ROWSTATS = 5,
+       K_EMBED = 6, K_STEPLOGIC = 7, K_CLASSES = 8 };
+
+template <typename F>
+void timed(cdsl_ctx* c, int cls, double bytes, double flops, F&& launch) {
+  if (!c->profiling) {
+    launch();
+    return;
+  }
+  while (c->ev_pool.size() < c->ev_used + 2) {
+    cudaEvent_t e;
+    cudaEventCreate(&e);
+    c->ev_pool.push_back(e);
+  }
+  const size_t ev = c->ev_used;
+  c->ev_used += 2;
+  cudaEventRecord(c->ev_pool[ev], c->stream);
+  launch();
+  cudaEventRecord(c->ev_pool[ev + 1], c->stream);
+  c->prof.push_back({cls, bytes, flops, ev});
+}
+
 void gemm(cdsl_ctx* c, const GemmArgs& a) {
   // bf16: the tensor-core kernel for every shape it supports (it streams weights faster than
   // the CUDA-core GEMV even at 4-8 rows); the weight-streaming GEMV otherwise at <= 8 rows;
   // float32 (and anything else): the CUDA-core tiled GEMM.
   const bool bf16 = c->dtype == CDSL_DTYPE_BF16;
-  const int impl = (bf16 && tc_supported(a)) ? 2 : (bf16 && a.R <= 8) ? 1 : 0;
-  size_t ev = 0;
-  if (c->profiling) {
-    while (c->ev_pool.size() < c->ev_used + 2) {
-      cudaEvent_t e;
-      cudaEventCreate(&e);
-      c->ev_pool.push_back(e);
-    }
-    ev = c->ev_used;
-    c->ev_used += 2;
-    cudaEventRecord(c->ev_pool[ev], c->stream);
-  }
-  if (impl == 1) {
-    launch_gemv(a, plan_gemv(a.K, a.n_virtual, kPlanSMs), c->gemv_part, c->gemv_cnt, c->stream);
-  } else if (impl == 2) {
+  const int impl = (bf16 && tc_supported(a)) ? K_GEMM_TC : (bf16 && a.R <= 8) ? K_GEMV : K_GEMM_SIMT;
+  double fl = 0;
+  const double by = c->profiling ? gemm_bytes(c, a, &fl) : 0.0;
+  if (impl == K_GEMV) {
+    timed(c, impl, by, fl, [&] {
+      launch_gemv(a, plan_gemv(a.K, a.n_virtual, kPlanSMs), c->gemv_part, c->gemv_cnt, c->stream);
+    });
+  } else if (impl == K_GEMM_TC) {
     TcMaps maps;
     for (int s = 0; s < 3; ++s) {
       const int seg = s < a.n_seg ? s : 0;
@@ -331,16 +349,10 @@ void gemm(cdsl_ctx* c, const GemmArgs& a) {
     const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(a.x);
     maps.xh = tensor_map(c, xb, a.ldx, c->R_pad, 16);
     maps.xl = tensor_map(c, xb + a.x_plane, a.ldx, c->R_pad, 16);
-    launch_gemm_tc(maps, a, plan_tc(a.K, a.n_virtual, a.R, kPlanSMs), c->gemv_part, c->gemv_cnt,
-                   c->stream);
+    const TcPlan p = plan_tc(a.K, a.n_virtual, a.R, kPlanSMs);
+    timed(c, impl, by, fl, [&] { launch_gemm_tc(maps, a, p, c->gemv_part, c->gemv_cnt, c->stream); });
   } else {
-    launch_gemm_simt(c->dtype, a, c->stream);
-  }
-  if (c->profiling) {
-    cudaEventRecord(c->ev_pool[ev + 1], c->stream);
-    double fl = 0;
-    const double by = gemm_bytes(c, a, &fl);
-    c->prof.push_back({impl, by, fl, ev});
+    timed(c, impl, by, fl, [&] { launch_gemm_simt(c->dtype, a, c->stream); });
   }
 }
 
@@ -400,11 +412,13 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     at.qb_count = (ap.rows_per_prompt * at.G + attn_qblock() - 1) / attn_qblock();
     n_z = c->B * at.qb_count;
   }
-  launch_embed(c->dtype, rows, R, m.embed, D, c->h, s);
+  timed(c, K_EMBED, 0, 0, [&] { launch_embed(c->dtype, rows, R, m.embed, D, c->h, s); });
   for (int l = 0; l < cfg.n_layers; ++l) {
     const auto& W = m.layers[l];
-    launch_rmsnorm(c->dtype, c->h, R, D, W[W_ATTN_NORM], cfg.norm_eps, c->X1, c->act_plane,
-                   nullptr, nullptr, nullptr, s);
+    timed(c, K_NORM, 0, 0, [&] {
+      launch_rmsnorm(c->dtype, c->h, R, D, W[W_ATTN_NORM], cfg.norm_eps, c->X1, c->act_plane,
+                     nullptr, nullptr, nullptr, s);
+    });
     GemmArgs q = gemm_base(c, m, EPI_QKV, D, c->X1, D, R);
     q.w[0] = W[W_Q]; q.w[1] = W[W_K]; q.w[2] = W[W_V];
     q.seg_rows[0] = H * hd; q.seg_rows[1] = KVH * hd; q.seg_rows[2] = KVH * hd;
@@ -416,13 +430,15 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     q.rope = m.rope;
     gemm(c, q);
     at.layer = l;
-    launch_attn(c->dtype, at, n_z, s);
+    timed(c, K_ATTN, 0, 0, [&] { launch_attn(c->dtype, at, n_z, s); });
     GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->X1, H * hd, R);
     o.w[0] = W[W_O]; o.seg_rows[0] = D; o.n_seg = 1; o.n_virtual = D;
     o.out_f32 = c->h; o.ld_out = D;
     gemm(c, o);
-    launch_rmsnorm(c->dtype, c->h, R, D, W[W_FFN_NORM], cfg.norm_eps, c->X1, c->act_plane,
-                   nullptr, nullptr, nullptr, s);
+    timed(c, K_NORM, 0, 0, [&] {
+      launch_rmsnorm(c->dtype, c->h, R, D, W[W_FFN_NORM], cfg.norm_eps, c->X1, c->act_plane,
+                     nullptr, nullptr, nullptr, s);
+    });
     GemmArgs g = gemm_base(c, m, EPI_SWIGLU, D, c->X1, D, R);
     g.w[0] = W[W_GATE]; g.w[1] = W[W_UP]; g.seg_rows[0] = F; g.seg_rows[1] = F; g.n_seg = 2;
     g.n_virtual = (F + 63) / 64 * 128;
@@ -435,8 +451,10 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     gemm(c, dn);
   }
   if (lm_rows > 0) {
-    launch_rmsnorm(c->dtype, c->h, lm_rows, D, m.final_norm, cfg.norm_eps, c->X1, c->act_plane,
-                   gather, head_out ? c->head_w : nullptr, head_out, s);
+    timed(c, K_NORM, 0, 0, [&] {
+      launch_rmsnorm(c->dtype, c->h, lm_rows, D, m.final_norm, cfg.norm_eps, c->X1, c->act_plane,
+                     gather, head_out ? c->head_w : nullptr, head_out, s);
+    });
     GemmArgs lm = gemm_base(c, m, EPI_STORE, D, c->X1, D, lm_rows);
     lm.w[0] = m.lm_head; lm.seg_rows[0] = cfg.vocab; lm.n_seg = 1; lm.n_virtual = cfg.vocab;
     lm.out_f32 = logits; lm.ld_out = cfg.vocab;
@@ -446,7 +464,7 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
 
 void do_lookahead(cdsl_ctx* c) {
   for (int j = 1; j <= c->d; ++j) {
-    launch_plan_draft(c->st, j, c->dft.spb, c->rows_d, c->stream);
+    timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_draft(c->st, j, c->dft.spb, c->rows_d, c->stream); });
     const int R = c->B * c->k + (j == 1 ? c->B : 0);
     AttnPass ap;
     ap.rows_per_prompt = c->k + (j == 1 ? 1 : 0);
@@ -455,12 +473,12 @@ void do_lookahead(cdsl_ctx* c) {
     a.logits = c->logits; a.R = c->B * c->k; a.V = c->V; a.k = c->k;
     a.x_out = c->st.x; a.logq_out = c->st.logq; a.out_stride = c->d; a.out_off = j - 1;
     a.status = c->st.status;
-    launch_row_stats(a, c->stream);
+    timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
   }
 }
 
 void do_verify(cdsl_ctx* c) {
-  launch_plan_verify(c->st, c->rows_v, c->stream);
+  timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_verify(c->st, c->rows_v, c->stream); });
   AttnPass ap;
   ap.rows_per_prompt = c->k * (c->d + 1);
   forward(c, c->tgt, c->rows_v, c->R_v, c->R_v, nullptr, c->logits,
@@ -469,14 +487,16 @@ void do_verify(cdsl_ctx* c) {
   a.logits = c->logits; a.R = c->R_v; a.V = c->V; a.k = c->k; a.dp1 = c->d + 1;
   a.next_x = c->st.x; a.amax = c->st.v_amax; a.logp = c->st.v_logp; a.topk = c->st.v_topk;
   a.status = c->st.status;
-  launch_row_stats(a, c->stream);
+  timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
 }
 
 void do_select(cdsl_ctx* c) {
-  launch_select(c->st, c->tgt.kv, c->dft.kv, 1, c->stream);
-  launch_commit_kv(c->st, c->tgt.kv, c->tgt.spb, 0, c->stream);
-  launch_commit_kv(c->st, c->dft.kv, c->dft.spb, 1, c->stream);
-  launch_advance(c->st, c->stream);
+  timed(c, K_STEPLOGIC, 0, 0, [&] {
+    launch_select(c->st, c->tgt.kv, c->dft.kv, 1, c->stream);
+    launch_commit_kv(c->st, c->tgt.kv, c->tgt.spb, 0, c->stream);
+    launch_commit_kv(c->st, c->dft.kv, c->dft.spb, 1, c->stream);
+    launch_advance(c->st, c->stream);
+  });
 }
 
 void copy_out(cdsl_ctx* c, void* dst, const void* src, size_t bytes) {

@@ -4,11 +4,12 @@
 // Prefix sharing: all rows of one prompt read the same prefix K/V. A block owns one prompt,
 // one KV head, one chunk of 64 prefix positions and 32 query vectors (query vector =
 // (row, query head of the GQA group)); it loads the chunk's K and V once into shared memory
-// and scores all its query vectors against them (split-KV, flash-decoding style). Each query
-// vector's partial result (max score m, sum of exponentials l, unnormalized output o) goes to
-// scratch; the last block of a (prompt, head, query block) to arrive merges the chunks in
-// order, adds the row's own tail keys (the beam's rows of this pass, causal within the beam)
-// and writes the normalized output in the GEMM-input format. fp32 throughout.
+// and scores all its query vectors against them (split-KV, flash-decoding style). One more
+// chunk per query block holds each row's own tail keys (its beam's rows of this pass, causal
+// within the beam). Each query vector's partial result (max score m, sum of exponentials l,
+// unnormalized output o) goes to scratch; the last block of a (prompt, head, query block) to
+// arrive merges the chunks in order (lanes over chunks, all loads in flight) and writes the
+// normalized output in the GEMM-input format. fp32 throughout.
 //
 // Score loop: a warp owns 4 query vectors (broadcast reads), its lanes own keys lane and
 // lane + 32 (rows of 132 floats: conflict-free 128-bit reads). Output loop: lanes own 4 (or 2)
@@ -43,8 +44,11 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
   __shared__ int s_wcnt[ATHREADS / 32];
   __shared__ int s_nrows, s_last;
   __shared__ float s_m[AQB], s_l[AQB];
+  __shared__ int s_page[ACH];
 
   const int chunk = blockIdx.x, g = blockIdx.y;
+  const int n_pchunks = gridDim.x - 1;          // prefix chunks; x == n_pchunks: tail keys
+  const bool tail_chunk = chunk == n_pchunks;
   int b, qb;
   if (a.zmap) {
     b = a.zmap[2 * blockIdx.z];
@@ -88,6 +92,8 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
     }
     __syncthreads();
   }
+  pdl_wait();                 // q, K/V and the scratch of the previous kernels are ready
+  pdl_launch_dependents();
   const int nq = min(AQB, s_nrows * G - qb * AQB);
   if (nq <= 0) return;   // no query vector in this block (no block of this group has any)
   int maxnp = 0;
@@ -96,7 +102,46 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
   float* po = a.part_o + (grp * gridDim.x + chunk) * AQB * HD;
   float* pml = a.part_ml + (grp * gridDim.x + chunk) * AQB * 2;
 
-  if (t0 < maxnp) {
+  constexpr int DPL = HD / 32;
+  if (tail_chunk) {
+    // ---- each row's own tail keys (at most 17): lanes over keys for the scores, over dims
+    //      for the output
+    for (int qi = warp; qi < nq; qi += ATHREADS / 32) {
+      const RowDesc rd = a.rows[s_row[qi]];
+      const int nt = min(rd.n_tail, 17);
+      const float* qrow = a.q + (size_t)s_row[qi] * H * HD + (size_t)(g * G + s_gg[qi]) * HD;
+      float sc = -INFINITY;
+      if (lane < nt) {
+        const float* kt = a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, rd.tail_base + lane, g);
+        float d = 0.f;
+#pragma unroll 8
+        for (int e = 0; e < HD; e += 4) {
+          const float4 qv = *reinterpret_cast<const float4*>(qrow + e);
+          const float4 kv = *reinterpret_cast<const float4*>(kt + e);
+          d += qv.x * kv.x + qv.y * kv.y + qv.z * kv.z + qv.w * kv.w;
+        }
+        sc = d * a.scale;
+      }
+      const float m = warp_max(sc);
+      const float pj = (lane < nt) ? expf(sc - m) : 0.f;
+      const float l = warp_sum(pj);
+      float o[DPL];
+#pragma unroll
+      for (int c = 0; c < DPL; ++c) o[c] = 0.f;
+      for (int j = 0; j < nt; ++j) {
+        const float w = __shfl_sync(0xffffffffu, pj, j);
+        const float* vt = a.kv.tail + kv_tail_offset(a.kv, a.layer, 1, rd.tail_base + j, g);
+#pragma unroll
+        for (int c = 0; c < DPL; ++c) o[c] = fmaf(w, vt[DPL * lane + c], o[c]);
+      }
+#pragma unroll
+      for (int c = 0; c < DPL; ++c) po[qi * HD + DPL * lane + c] = o[c];
+      if (lane == 0) {
+        pml[2 * qi] = (nt > 0) ? m : -INFINITY;
+        pml[2 * qi + 1] = l;
+      }
+    }
+  } else if (t0 < maxnp) {
     // ---- stage Q (scaled), K and V of positions t0 .. t0 + ACH - 1
     for (int idx = threadIdx.x; idx < AQB * (HD / 4); idx += ATHREADS) {
       const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
@@ -108,23 +153,35 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
       }
       *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
     }
-    const int* pt = a.kv.page_table + b * a.kv.max_pages;
+    // page ids of this chunk's positions (a chunk spans 64 / page_size pages, at least one)
     const int pmask = (1 << a.kv.page_shift) - 1;
-    for (int idx = threadIdx.x; idx < ACH * (HD / 4); idx += ATHREADS) {
+    if (threadIdx.x < ACH) {
+      const int t = t0 + threadIdx.x;
+      s_page[threadIdx.x] =
+          (t < maxnp) ? a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)] : -1;
+    }
+    __syncthreads();
+    // every thread first issues all of its K and V loads, then stores them
+    constexpr int PER = ACH * (HD / 4) / ATHREADS;   // float4 per thread per matrix
+    float4 kr[PER], vr[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int idx = threadIdx.x + i * ATHREADS;
       const int j = idx / (HD / 4), e4 = idx % (HD / 4);
-      const int t = t0 + j;
-      float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
-      if (t < maxnp) {
-        const int page = pt[t >> a.kv.page_shift];
-        if (page >= 0) {
-          const size_t ko = kv_prefix_offset(a.kv, a.layer, page, 0, g, t & pmask) + 4 * e4;
-          const size_t vo = kv_prefix_offset(a.kv, a.layer, page, 1, g, t & pmask) + 4 * e4;
-          kv = *reinterpret_cast<const float4*>(a.kv.pool + ko);
-          vv = *reinterpret_cast<const float4*>(a.kv.pool + vo);
-        }
+      const int page = s_page[j];
+      kr[i] = vr[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (page >= 0) {
+        const size_t ko = kv_prefix_offset(a.kv, a.layer, page, 0, g, (t0 + j) & pmask) + 4 * e4;
+        kr[i] = __ldg(reinterpret_cast<const float4*>(a.kv.pool + ko));
+        vr[i] = __ldg(reinterpret_cast<const float4*>(a.kv.pool + ko + ((size_t)a.kv.kvh << a.kv.page_shift) * HD));
       }
-      *reinterpret_cast<float4*>(kS + j * L::QP + 4 * e4) = kv;
-      *reinterpret_cast<float4*>(vS + j * HD + 4 * e4) = vv;
+    }
+#pragma unroll
+    for (int i = 0; i < PER; ++i) {
+      const int idx = threadIdx.x + i * ATHREADS;
+      const int j = idx / (HD / 4), e4 = idx % (HD / 4);
+      *reinterpret_cast<float4*>(kS + j * L::QP + 4 * e4) = kr[i];
+      *reinterpret_cast<float4*>(vS + j * HD + 4 * e4) = vr[i];
     }
     __syncthreads();
 
@@ -163,7 +220,6 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
     __syncwarp();
 
     // ---- partial output: lane -> dims [DPL*lane, DPL*lane + DPL)
-    constexpr int DPL = HD / 32;
     float o[4][DPL];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
@@ -205,62 +261,74 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  constexpr int DPL = HD / 32;
-  for (int qi = warp; qi < nq; qi += ATHREADS / 32) {
-    const int r = s_row[qi], gg = s_gg[qi];
-    const RowDesc rd = a.rows[r];
-    const int ncv = (rd.n_prefix + ACH - 1) / ACH;
-    const float* qrow = a.q + (size_t)r * H * HD + (size_t)(g * G + gg) * HD;
+  // (1) per query vector: max over its chunks and the softmax weight of every chunk
+  constexpr int MAXP = 64;   // prefix chunks + the tail chunk (n_chunks <= 63, checked on the host)
+  float* wS = pS;            // [AQB][MAXP] reuses the probability tile (ACH * AQB floats)
+  static_assert(AQB * MAXP <= ACH * AQB, "merge weights fit in the probability tile");
+  for (int i = threadIdx.x; i < nq * MAXP; i += ATHREADS) {
+    const int qi = i / MAXP, j = i % MAXP;
+    const int ncv = (s_np[qi] + ACH - 1) / ACH;
+    float mc = -INFINITY;
+    if (j <= ncv) {
+      const int cj = j < ncv ? j : n_pchunks;
+      mc = __ldcg(a.part_ml + ((grp * gridDim.x + cj) * AQB + qi) * 2);
+    }
+    wS[i] = mc;
+  }
+  __syncthreads();
+  if (threadIdx.x < nq) {
+    const int qi = threadIdx.x;
+    const int ncv = (s_np[qi] + ACH - 1) / ACH;
     float m = -INFINITY;
-    for (int c = 0; c < ncv; ++c)
-      m = fmaxf(m, __ldcg(a.part_ml + ((grp * gridDim.x + c) * AQB + qi) * 2));
-    // tail keys of the row's beam (at most 17)
-    float ts[17];
-    const int nt = min(rd.n_tail, 17);
-    for (int j = 0; j < nt; ++j) {
-      const float* kt = a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, rd.tail_base + j, g);
-      float d = 0.f;
-      for (int e = lane; e < HD; e += 32) d += qrow[e] * kt[e];
-      d = warp_sum(d) * a.scale;
-      ts[j] = d;
-      m = fmaxf(m, d);
+    for (int j = 0; j <= ncv; ++j) m = fmaxf(m, wS[qi * MAXP + j]);
+    float l = 0.f;
+    for (int j = 0; j <= ncv; ++j) {
+      const float mc = wS[qi * MAXP + j];
+      const int cj = j < ncv ? j : n_pchunks;
+      const float w = (mc > -INFINITY) ? expf(mc - m) : 0.f;
+      l += w * __ldcg(a.part_ml + ((grp * gridDim.x + cj) * AQB + qi) * 2 + 1);
+      wS[qi * MAXP + j] = w;
     }
-    float l = 0.f, o[DPL];
-#pragma unroll
-    for (int c = 0; c < DPL; ++c) o[c] = 0.f;
-    for (int c = 0; c < ncv; ++c) {
-      const size_t base = (grp * gridDim.x + c) * AQB + qi;
-      const float w = expf(__ldcg(a.part_ml + base * 2) - m);
-      l += w * __ldcg(a.part_ml + base * 2 + 1);
-#pragma unroll
-      for (int cc = 0; cc < DPL; ++cc) o[cc] += w * __ldcg(a.part_o + base * HD + DPL * lane + cc);
-    }
-    for (int j = 0; j < nt; ++j) {
-      const float w = expf(ts[j] - m);
-      const float* vt = a.kv.tail + kv_tail_offset(a.kv, a.layer, 1, rd.tail_base + j, g);
-      l += w;
-#pragma unroll
-      for (int cc = 0; cc < DPL; ++cc) o[cc] += w * vt[DPL * lane + cc];
-    }
-    const float inv = 1.0f / l;
+    s_l[qi] = 1.0f / l;
+  }
+  __syncthreads();
+  // (2) outputs: items (query vector, 4 dims), every item's chunk loads in flight together
+  {
     T* out = reinterpret_cast<T*>(a.out);
-#pragma unroll
-    for (int cc = 0; cc < DPL; ++cc)
-      store_act<T>(out, a.plane, (size_t)r * H * HD + (size_t)(g * G + gg) * HD + DPL * lane + cc,
-                   o[cc] * inv);
+    for (int i = threadIdx.x; i < nq * (HD / 4); i += ATHREADS) {
+      const int qi = i / (HD / 4), e4 = i % (HD / 4);
+      const int ncv = (s_np[qi] + ACH - 1) / ACH;
+      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+      for (int j = 0; j <= ncv; ++j) {
+        const int cj = j < ncv ? j : n_pchunks;
+        const float w = wS[qi * MAXP + j];
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(
+            a.part_o + ((grp * gridDim.x + cj) * AQB + qi) * HD + 4 * e4));
+        o.x = fmaf(w, v.x, o.x); o.y = fmaf(w, v.y, o.y);
+        o.z = fmaf(w, v.z, o.z); o.w = fmaf(w, v.w, o.w);
+      }
+      const float inv = s_l[qi];
+      const size_t dst = (size_t)s_row[qi] * H * HD + (size_t)(g * G + s_gg[qi]) * HD + 4 * e4;
+      store_act<T>(out, a.plane, dst + 0, o.x * inv);
+      store_act<T>(out, a.plane, dst + 1, o.y * inv);
+      store_act<T>(out, a.plane, dst + 2, o.z * inv);
+      store_act<T>(out, a.plane, dst + 3, o.w * inv);
+    }
   }
   if (threadIdx.x == 0) a.cnt[grp] = 0;
 }
 
 template <typename T, int HD>
 void launch_t(const AttnArgs& a, int n_z, cudaStream_t s) {
-  dim3 grid(a.n_chunks, a.kv.kvh, n_z);
-  k_attn<T, HD><<<grid, ATHREADS, AttnSmem<HD>::bytes, s>>>(a);
+  dim3 grid(a.n_chunks + 1, a.kv.kvh, n_z);   // + the tail-key chunk
+  launch_pdl(k_attn<T, HD>, grid, dim3(ATHREADS), AttnSmem<HD>::bytes, s, a);
 }
 
 }  // namespace
 
 int attn_chunk() { return ACH; }
+int attn_max_chunks() { return 63; }
 int attn_qblock() { return AQB; }
 
 int configure_attention() {

@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
-  if (threadIdx.x == 0) pdl_launch_dependents();
+  pdl_launch_dependents();
   const uint32_t tmem = tmem_base;
 
   if (warp == 0) {
@@ -407,17 +407,7 @@ int configure_gemm_tc() {
 
 void launch_gemm_tc(const TcMaps& maps, const GemmArgs& a, const TcPlan& p, float* part,
                     int* tile_cnt, cudaStream_t s) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.ctas);
-  cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = p.smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaLaunchKernelEx(&cfg, k_gemm_tc, maps, a, p, part, tile_cnt);
+  launch_pdl(k_gemm_tc, dim3(p.ctas), dim3(kThreads), p.smem, s, maps, a, p, part, tile_cnt);
 }
 
 }  // namespace cdsl

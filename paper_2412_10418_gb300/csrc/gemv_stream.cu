@@ -72,6 +72,8 @@ __device__ __forceinline__ void transpose_reduce(float (&v)[NV]) {
 template <int RM>
 __global__ void __launch_bounds__(THREADS) k_gemv(GemmArgs a, int k_split, int n_splits,
                                                  float* part, int* tile_cnt) {
+  pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ float4 smem4[];
   float* xs = reinterpret_cast<float*>(smem4);   // [RM][k_split]
   float* tile = xs + RM * k_split;                // [RM][TV]

@@ -40,6 +40,8 @@ __device__ unsigned long long block_max_u64(unsigned long long v, unsigned long 
 // ------------------------------------------------------------------------------ embedding
 template <typename T>
 __global__ void k_embed(const RowDesc* rows, const T* E, int D, float* h) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int r = blockIdx.x;
   const T* e = E + (size_t)rows[r].token * D;
   for (int c = threadIdx.x; c < D; c += blockDim.x) h[(size_t)r * D + c] = to_f32<T>(e[c]);
@@ -51,6 +53,8 @@ __global__ void k_embed(const RowDesc* rows, const T* E, int D, float* h) {
 template <typename T>
 __global__ void k_rmsnorm(const float* h, int D, const T* g, float eps, T* out, size_t plane,
                           const int32_t* gather, const float* head_w, float* head_out) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ float red[kMaxWarps];
   const int r = blockIdx.x;
   const int src = gather ? gather[r] : r;
@@ -73,6 +77,8 @@ __global__ void k_rmsnorm(const float* h, int D, const T* g, float eps, T* out, 
 
 // ------------------------------------------------------------------------------ row stats
 __global__ void k_row_stats(RowStatsArgs a) {
+  pdl_wait();
+  pdl_launch_dependents();
   __shared__ unsigned long long redk[kMaxWarps];
   __shared__ float red[kMaxWarps];
   __shared__ int bad_s;
@@ -137,6 +143,8 @@ __global__ void k_row_stats(RowStatsArgs a) {
 // see the prefix and their own tail slots 0..j-1. Call 1 adds one row per prompt: the pending
 // token L-1 of a fully accepted step, written straight into the draft prefix pages.
 __global__ void k_plan_draft(StepState st, int j, int spb, RowDesc* rows) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   const int nbk = st.B * st.k;
   if (r < nbk) {
@@ -178,6 +186,8 @@ __global__ void k_plan_draft(StepState st, int j, int spb, RowDesc* rows) {
 // Verify rows (b, i, j), j = 0..d: token c_bi (j = 0) or x_bi,j at position L + j; they see
 // the prefix and their beam's tail slots 0..j (causal within the beam, nothing across beams).
 __global__ void k_plan_verify(StepState st, RowDesc* rows) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int dp1 = st.d + 1;
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= st.B * st.k * dp1) return;
@@ -212,6 +222,8 @@ __device__ void alloc_pages(const KvStore& kv, int b, int from, int to, int32_t*
 
 // One warp per prompt, one lane per beam: n_b, rewards, b*, state, emission, page allocation.
 __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int b = blockIdx.x, lane = threadIdx.x;
   const int k = st.k, d = st.d, dp1 = d + 1;
   if (st.gen[b] >= st.max_new) {
@@ -284,6 +296,8 @@ __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
 
 // Copy the winner's tail K/V rows 0..cnt-1 to prefix positions L..L+cnt-1.
 __global__ void k_commit_kv(StepState st, KvStore kv, int spb, int is_draft) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int b = blockIdx.x, layer = blockIdx.y, kvsel = blockIdx.z;
   int cnt = st.n_emit[b];
   if (is_draft) cnt = min(cnt, st.d);
@@ -303,6 +317,8 @@ __global__ void k_commit_kv(StepState st, KvStore kv, int spb, int is_draft) {
 
 // pfx <- pfx + O, T <- T + O; the next beams are the top-k of the winner's row cnt-1.
 __global__ void k_advance(StepState st) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int b = blockIdx.x, lane = threadIdx.x;
   const int k = st.k, d = st.d, dp1 = d + 1;
   if (b == 0 && lane == 0) {
@@ -361,40 +377,42 @@ __global__ void k_rope_table(float2* table, int n_pos, int hd, double theta) {
 
 void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int D, float* h,
                   cudaStream_t s) {
-  DISPATCH(dtype, k_embed<T><<<R, 256, 0, s>>>(rows, (const T*)embed, D, h));
+  DISPATCH(dtype, launch_pdl(k_embed<T>, dim3(R), dim3(256), 0, s, rows, (const T*)embed, D, h));
 }
 
 void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
                     void* out, size_t plane, const int32_t* gather, const float* head_w,
                     float* head_out, cudaStream_t s) {
-  DISPATCH(dtype, k_rmsnorm<T><<<R, 256, 0, s>>>(h, D, (const T*)gain, eps, (T*)out, plane,
-                                                 gather, head_w, head_out));
+  DISPATCH(dtype, launch_pdl(k_rmsnorm<T>, dim3(R), dim3(256), 0, s, h, D, (const T*)gain, eps,
+                             (T*)out, plane, gather, head_w, head_out));
 }
 
 void launch_row_stats(const RowStatsArgs& a, cudaStream_t s) {
-  k_row_stats<<<a.R, 512, 0, s>>>(a);
+  launch_pdl(k_row_stats, dim3(a.R), dim3(512), 0, s, a);
 }
 
 void launch_plan_draft(const StepState& st, int j, int spb, RowDesc* rows, cudaStream_t s) {
   const int n = st.B * st.k + (j == 1 ? st.B : 0);
-  k_plan_draft<<<(n + 127) / 128, 128, 0, s>>>(st, j, spb, rows);
+  launch_pdl(k_plan_draft, dim3((n + 127) / 128), dim3(128), 0, s, st, j, spb, rows);
 }
 
 void launch_plan_verify(const StepState& st, RowDesc* rows, cudaStream_t s) {
   const int n = st.B * st.k * (st.d + 1);
-  k_plan_verify<<<(n + 127) / 128, 128, 0, s>>>(st, rows);
+  launch_pdl(k_plan_verify, dim3((n + 127) / 128), dim3(128), 0, s, st, rows);
 }
 
 void launch_select(const StepState& st, KvStore tkv, KvStore dkv, int commit, cudaStream_t s) {
-  k_select<<<st.B, 32, 0, s>>>(st, tkv, dkv, commit);
+  launch_pdl(k_select, dim3(st.B), dim3(32), 0, s, st, tkv, dkv, commit);
 }
 
 void launch_commit_kv(const StepState& st, KvStore kv, int spb, int is_draft, cudaStream_t s) {
   dim3 grid(st.B, kv.n_layers, 2);
-  k_commit_kv<<<grid, 256, 0, s>>>(st, kv, spb, is_draft);
+  launch_pdl(k_commit_kv, grid, dim3(256), 0, s, st, kv, spb, is_draft);
 }
 
-void launch_advance(const StepState& st, cudaStream_t s) { k_advance<<<st.B, 32, 0, s>>>(st); }
+void launch_advance(const StepState& st, cudaStream_t s) {
+  launch_pdl(k_advance, dim3(st.B), dim3(32), 0, s, st);
+}
 
 void launch_rope_table(float2* table, int n_pos, int hd, float theta, cudaStream_t s) {
   const int n = n_pos * (hd / 2);

@@ -45,11 +45,11 @@ void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int 
 void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
                     void* out, size_t plane, const int32_t* gather, const float* head_w,
                     float* head_out, cudaStream_t s);
-// Attention of a pass (attention.cu). Blocks: (prefix chunk of attn_chunk() positions, kv
-// head, z) with z -> (prompt, query block of attn_qblock() query vectors) either dense
-// (b = z / qb_count) or from zmap[2z], zmap[2z+1]. Scratch: part_o
-// [n_z][kvh][n_chunks][qblock][hd], part_ml [n_z][kvh][n_chunks][qblock][2], cnt [n_z][kvh]
-// (zero between launches).
+// Attention of a pass (attention.cu). Blocks: (prefix chunk of attn_chunk() positions or the
+// tail-key chunk, kv head, z) with z -> (prompt, query block of attn_qblock() query vectors)
+// either dense (b = z / qb_count) or from zmap[2z], zmap[2z+1]. Scratch: part_o
+// [n_z][kvh][n_chunks + 1][qblock][hd], part_ml [n_z][kvh][n_chunks + 1][qblock][2],
+// cnt [n_z][kvh] (zero between launches).
 struct AttnArgs {
   const float* q; int32_t n_heads, G;
   KvStore kv; int32_t layer;
@@ -60,6 +60,7 @@ struct AttnArgs {
   float* part_o; float* part_ml; int32_t* cnt;
 };
 int attn_chunk();
+int attn_max_chunks();
 int attn_qblock();
 int configure_attention();
 void launch_attn(int dtype, const AttnArgs& a, int n_z, cudaStream_t s);
