@@ -131,7 +131,9 @@ int check_model(const cdsl_model_cfg* m, const char* name, std::string* why) {
     return bad("n_heads must be a positive multiple of n_kv_heads");
   if (m->n_heads / m->n_kv_heads > 16) return bad("more than 16 query heads per kv head");
   if (m->d_ffn < 8 || m->d_ffn % 8) return bad("d_ffn must be a positive multiple of 8");
-  if (m->vocab < 2 || m->vocab % 8) return bad("vocab must be a multiple of 8");
+  if (m->vocab < 2 || m->vocab % 8 || m->vocab > 32768)
+    return bad("vocab must be a multiple of 8, at most 32768");
+  if (m->d_model > 8192) return bad("d_model must be at most 8192");
   if (m->dtype != CDSL_DTYPE_F32 && m->dtype != CDSL_DTYPE_BF16) return bad("unknown dtype");
   if (!(m->rope_theta > 0.f) || !(m->norm_eps > 0.f)) return bad("rope_theta and norm_eps must be > 0");
   return CDSL_OK;

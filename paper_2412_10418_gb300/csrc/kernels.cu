@@ -51,23 +51,40 @@ __global__ void k_embed(const RowDesc* rows, const T* E, int D, float* h) {
 // out[r] = h[src] / sqrt(mean(h[src]^2) + eps) * g, src = gather ? gather[r] : r.
 // With head_w: head_out[r] = sigmoid(head_w . normalized row) (fp32, before rounding).
 template <typename T>
-__global__ void k_rmsnorm(const float* h, int D, const T* g, float eps, T* out, size_t plane,
-                          const int32_t* gather, const float* head_w, float* head_out) {
+__global__ void __launch_bounds__(256) k_rmsnorm(const float* h, int D, const T* g, float eps,
+                                                T* out, size_t plane, const int32_t* gather,
+                                                const float* head_w, float* head_out) {
   pdl_wait();
   pdl_launch_dependents();
   __shared__ float red[kMaxWarps];
+  constexpr int MAXV = 8;   // float4 per thread: D <= 8 * 4 * 256 = 8192
   const int r = blockIdx.x;
   const int src = gather ? gather[r] : r;
-  const float* x = h + (size_t)src * D;
+  const float4* x = reinterpret_cast<const float4*>(h + (size_t)src * D);
+  const int n4 = D >> 2;
+  float4 v[MAXV];
   float ss = 0.f;
-  for (int c = threadIdx.x; c < D; c += blockDim.x) ss += x[c] * x[c];
+#pragma unroll
+  for (int i = 0; i < MAXV; ++i) {
+    const int c = threadIdx.x + i * 256;
+    v[i] = c < n4 ? x[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+#pragma unroll
+  for (int i = 0; i < MAXV; ++i) ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
   ss = block_sum(ss, red);
   const float inv = rsqrtf(ss / (float)D + eps);
   float hw = 0.f;
-  for (int c = threadIdx.x; c < D; c += blockDim.x) {
-    const float y = x[c] * inv * to_f32<T>(g[c]);
-    store_act<T>(out, plane, (size_t)r * D + c, y);
-    if (head_w) hw += head_w[c] * y;
+#pragma unroll
+  for (int i = 0; i < MAXV; ++i) {
+    const int c = threadIdx.x + i * 256;
+    if (c >= n4) continue;
+    const float e[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float y = e[q] * inv * to_f32<T>(g[4 * c + q]);
+      store_act<T>(out, plane, (size_t)r * D + 4 * c + q, y);
+      if (head_w) hw += head_w[4 * c + q] * y;
+    }
   }
   if (head_w) {
     hw = block_sum(hw, red);
@@ -76,30 +93,54 @@ __global__ void k_rmsnorm(const float* h, int D, const T* g, float eps, T* out, 
 }
 
 // ------------------------------------------------------------------------------ row stats
-__global__ void k_row_stats(RowStatsArgs a) {
+// One block per logits row; each thread holds its slice of the row in registers (one load
+// pass), then max / argmax, log-sum-exp and the top-k passes run on the registers.
+constexpr int RS_THREADS = 512;
+constexpr int RS_MAXV = 16;   // float4 per thread: V <= 16 * 4 * 512 = 32768
+
+__global__ void __launch_bounds__(RS_THREADS) k_row_stats(RowStatsArgs a) {
   pdl_wait();
   pdl_launch_dependents();
   __shared__ unsigned long long redk[kMaxWarps];
   __shared__ float red[kMaxWarps];
   __shared__ int bad_s;
   const int r = blockIdx.x;
-  const float* v = a.logits + (size_t)r * a.V;
+  const float* row = a.logits + (size_t)r * a.V;
+  const float4* v4 = reinterpret_cast<const float4*>(row);
+  const int n4 = a.V >> 2;
   if (threadIdx.x == 0) bad_s = 0;
+  float4 x[RS_MAXV];
+#pragma unroll
+  for (int i = 0; i < RS_MAXV; ++i) {
+    const int c = threadIdx.x + i * RS_THREADS;
+    x[i] = c < n4 ? v4[c] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+  }
   __syncthreads();
   unsigned long long best = 0;
   int bad = 0;
-  for (int i = threadIdx.x; i < a.V; i += blockDim.x) {
-    const float x = v[i];
-    if (!isfinite(x)) bad = 1;
-    const unsigned long long key = argmax_key(x, i);
-    best = key > best ? key : best;
+#pragma unroll
+  for (int i = 0; i < RS_MAXV; ++i) {
+    const int c = threadIdx.x + i * RS_THREADS;
+    if (c >= n4) continue;
+    const float e[4] = {x[i].x, x[i].y, x[i].z, x[i].w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (!isfinite(e[q])) bad = 1;
+      const unsigned long long key = argmax_key(e[q], 4 * c + q);
+      best = key > best ? key : best;
+    }
   }
   if (bad) atomicOr(&bad_s, 1);
   best = block_max_u64(best, redk);
   const int amax = argmax_key_index(best);
-  const float m = v[amax];
+  const float m = row[amax];
   float z = 0.f;
-  for (int i = threadIdx.x; i < a.V; i += blockDim.x) z += expf(v[i] - m);
+#pragma unroll
+  for (int i = 0; i < RS_MAXV; ++i) {
+    const int c = threadIdx.x + i * RS_THREADS;
+    if (c >= n4) continue;
+    z += expf(x[i].x - m) + expf(x[i].y - m) + expf(x[i].z - m) + expf(x[i].w - m);
+  }
   z = block_sum(z, red);
   const float lse = m + logf(z);
   if (threadIdx.x == 0 && bad_s) set_status(a.status, CDSL_ENONFINITE);
@@ -116,7 +157,7 @@ __global__ void k_row_stats(RowStatsArgs a) {
     const int j = r % a.dp1, bi = r / a.dp1, d = a.dp1 - 1;
     if (j < d && a.logp) {
       const int tok = a.next_x[bi * d + j];
-      a.logp[bi * d + j] = v[tok] - lse;
+      a.logp[bi * d + j] = row[tok] - lse;
     }
   }
   if (a.topk) {
@@ -127,9 +168,16 @@ __global__ void k_row_stats(RowStatsArgs a) {
     if (threadIdx.x == 0) a.topk[dst * a.k] = amax;
     for (int p = 1; p < a.k; ++p) {
       unsigned long long cur = 0;
-      for (int i = threadIdx.x; i < a.V; i += blockDim.x) {
-        const unsigned long long key = argmax_key(v[i], i);
-        if (key < prev && key > cur) cur = key;
+#pragma unroll
+      for (int i = 0; i < RS_MAXV; ++i) {
+        const int c = threadIdx.x + i * RS_THREADS;
+        if (c >= n4) continue;
+        const float e[4] = {x[i].x, x[i].y, x[i].z, x[i].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const unsigned long long key = argmax_key(e[q], 4 * c + q);
+          if (key < prev && key > cur) cur = key;
+        }
       }
       cur = block_max_u64(cur, redk);
       if (threadIdx.x == 0) a.topk[dst * a.k + p] = argmax_key_index(cur);
@@ -388,7 +436,7 @@ void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, f
 }
 
 void launch_row_stats(const RowStatsArgs& a, cudaStream_t s) {
-  launch_pdl(k_row_stats, dim3(a.R), dim3(512), 0, s, a);
+  launch_pdl(k_row_stats, dim3(a.R), dim3(RS_THREADS), 0, s, a);
 }
 
 void launch_plan_draft(const StepState& st, int j, int spb, RowDesc* rows, cudaStream_t s) {
