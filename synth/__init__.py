@@ -127,7 +127,17 @@ THIRTEEN_B = Workload(
     batch=4, prompt_len=1024, prompt_dist="zipf", k=8, d=6, max_new=256, n_keywords=5,
     reward_head=True)
 
-WORKLOADS: Dict[str, Workload] = {w.name: w for w in (TINY, SMALL, SEVEN_B, THIRTEEN_B)}
+# Two layers of each 7B-shaped model: the same projection shapes (the gate/up weights alone,
+# 180 MB, exceed the 129 MB L2) in about 1 GB of device memory, for kernel profiling captures.
+SEVEN_B_SLICE = Workload(
+    name="7b-2layer-bf16", dtype=DTYPE_BF16,
+    target=dataclasses.replace(SEVEN_B.target, n_layers=2),
+    draft=dataclasses.replace(DRAFT_1B, n_layers=2),
+    batch=1, prompt_len=512, prompt_dist="zipf", k=4, d=4, max_new=128, n_keywords=5,
+    reward_head=True)
+
+WORKLOADS: Dict[str, Workload] = {w.name: w for w in (TINY, SMALL, SEVEN_B, THIRTEEN_B,
+                                                      SEVEN_B_SLICE)}
 
 
 def scaled(w: Workload, **changes) -> Workload:
@@ -227,7 +237,7 @@ def model_weights(w: Workload, which: str, device: str = "host"):
     are drawn on the GPU."""
     shape = w.target if which == "target" else w.draft
     stream = _STREAM_TARGET if which == "target" else _STREAM_DRAFT
-    big = shape.n_params() > 400_000_000
+    big = shape.n_params() > 400_000_000 or shape.d_model >= 2048
     if device == "host":
         if big:
             raise ValueError("7B/13B-sized weights are drawn on the GPU; use device='cuda' then to_host()")
