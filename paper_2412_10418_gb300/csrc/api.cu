@@ -65,6 +65,10 @@ struct cdsl_ctx {
   float* h = nullptr;
   void* X1 = nullptr;
   void* X2 = nullptr;
+  void* Xa = nullptr;           // attention output (input of the O projection)
+  float* ss_a = nullptr;        // partial sums of h^2 (RMSNorm row scales), two ping-pong sets
+  float* ss_b = nullptr;
+  float* ss_hw = nullptr;       // reward-head partial sums
   float* qbuf = nullptr;
   float* logits = nullptr;
   RowDesc* rows_d = nullptr;
@@ -210,6 +214,11 @@ size_t carve(cdsl_ctx* c, void* base) {
   c->act_plane = (size_t)c->R_pad * c->act_cols;
   c->X1 = cv.take<float>(c->act_plane);
   c->X2 = cv.take<float>(c->act_plane);
+  c->Xa = cv.take<float>(c->act_plane);
+  const size_t ss_n = (size_t)(c->d_max / 32) * c->R_pad;
+  c->ss_a = cv.take<float>(ss_n);
+  c->ss_b = cv.take<float>(ss_n);
+  c->ss_hw = cv.take<float>(ss_n);
   c->qbuf = cv.take<float>((size_t)c->R_pad * c->q_cols);
   const int lm_rows = std::max(c->R_v, std::max(B * k, B));
   c->logits = cv.take<float>((size_t)lm_rows * c->V);
@@ -394,15 +403,20 @@ struct AttnPass {
   int n_chunks = 0;
 };
 
+// One forward pass of a model over R rows described by `rows`; for lm_rows > 0 the final
+// norm + LM head run over rows gather[i] (or the first lm_rows rows) into logits. RMSNorm is
+// folded into the GEMMs (the residual epilogues write h . g_next and the partial sums of h^2,
+// the consumers scale by the row factor); only a gathered LM input is normalized by a kernel.
+// With want_head, the last layer also leaves the reward-head partials in c->ss_hw.
 void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
-             const int32_t* gather, float* logits, float* head_out, const AttnPass& ap) {
+             const int32_t* gather, float* logits, bool want_head, const AttnPass& ap) {
   const cdsl_model_cfg& cfg = m.cfg;
   const int D = cfg.d_model, hd = cfg.head_dim, H = cfg.n_heads, KVH = cfg.n_kv_heads;
-  const int F = cfg.d_ffn;
+  const int F = cfg.d_ffn, L = cfg.n_layers;
   cudaStream_t s = c->stream;
   AttnArgs at{};
   at.q = c->qbuf; at.n_heads = H; at.G = H / KVH; at.kv = m.kv; at.rows = rows; at.R = R;
-  at.out = c->X1; at.plane = c->act_plane; at.scale = 1.0f / sqrtf((float)hd);
+  at.out = c->Xa; at.plane = c->act_plane; at.scale = 1.0f / sqrtf((float)hd);
   at.n_chunks = ap.n_chunks ? ap.n_chunks : c->attn_chunks;
   at.part_o = c->attn_o; at.part_ml = c->attn_ml; at.cnt = c->attn_cnt;
   int n_z;
@@ -414,13 +428,21 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     at.qb_count = (ap.rows_per_prompt * at.G + attn_qblock() - 1) / attn_qblock();
     n_z = c->B * at.qb_count;
   }
-  timed(c, K_EMBED, 0, 0, [&] { launch_embed(c->dtype, rows, R, m.embed, D, c->h, s); });
-  for (int l = 0; l < cfg.n_layers; ++l) {
+  const int ld_ss = c->R_pad;
+  auto normed_input = [&](GemmArgs& a, const float* ss) {
+    a.in_ss = ss; a.norm_D = D; a.ld_ss = ld_ss; a.norm_eps = cfg.norm_eps;
+  };
+  auto residual_out = [&](GemmArgs& a, const void* g_next, float* ss_out, bool head) {
+    a.out_f32 = c->h; a.ld_out = D;
+    a.next_x = c->X1; a.next_g = g_next; a.out_ss = ss_out; a.ld_ss = ld_ss;
+    if (head) { a.head_w = c->head_w; a.out_hw = c->ss_hw; }
+  };
+  timed(c, K_EMBED, 0, 0, [&] {
+    launch_embed(c->dtype, rows, R, m.embed, D, c->h, c->X1, c->act_plane,
+                 m.layers[0][W_ATTN_NORM], c->ss_a, ld_ss, s);
+  });
+  for (int l = 0; l < L; ++l) {
     const auto& W = m.layers[l];
-    timed(c, K_NORM, 0, 0, [&] {
-      launch_rmsnorm(c->dtype, c->h, R, D, W[W_ATTN_NORM], cfg.norm_eps, c->X1, c->act_plane,
-                     nullptr, nullptr, nullptr, s);
-    });
     GemmArgs q = gemm_base(c, m, EPI_QKV, D, c->X1, D, R);
     q.w[0] = W[W_Q]; q.w[1] = W[W_K]; q.w[2] = W[W_V];
     q.seg_rows[0] = H * hd; q.seg_rows[1] = KVH * hd; q.seg_rows[2] = KVH * hd;
@@ -430,36 +452,40 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     q.layer = l;
     q.rows = rows;
     q.rope = m.rope;
+    normed_input(q, c->ss_a);
     gemm(c, q);
     at.layer = l;
     timed(c, K_ATTN, 0, 0, [&] { launch_attn(c->dtype, at, n_z, s); });
-    GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->X1, H * hd, R);
+    GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->Xa, H * hd, R);
     o.w[0] = W[W_O]; o.seg_rows[0] = D; o.n_seg = 1; o.n_virtual = D;
-    o.out_f32 = c->h; o.ld_out = D;
+    residual_out(o, W[W_FFN_NORM], c->ss_b, false);
     gemm(c, o);
-    timed(c, K_NORM, 0, 0, [&] {
-      launch_rmsnorm(c->dtype, c->h, R, D, W[W_FFN_NORM], cfg.norm_eps, c->X1, c->act_plane,
-                     nullptr, nullptr, nullptr, s);
-    });
     GemmArgs g = gemm_base(c, m, EPI_SWIGLU, D, c->X1, D, R);
     g.w[0] = W[W_GATE]; g.w[1] = W[W_UP]; g.seg_rows[0] = F; g.seg_rows[1] = F; g.n_seg = 2;
     g.n_virtual = (F + 63) / 64 * 128;
     g.d_ffn = F;
     g.out_act = c->X2; g.ld_act = F;
+    normed_input(g, c->ss_b);
     gemm(c, g);
     GemmArgs dn = gemm_base(c, m, EPI_RESID, F, c->X2, F, R);
     dn.w[0] = W[W_DOWN]; dn.seg_rows[0] = D; dn.n_seg = 1; dn.n_virtual = D;
-    dn.out_f32 = c->h; dn.ld_out = D;
+    const bool last = l + 1 == L;
+    residual_out(dn, last ? m.final_norm : m.layers[l + 1][W_ATTN_NORM], c->ss_a,
+                 last && want_head && c->head_w);
     gemm(c, dn);
   }
   if (lm_rows > 0) {
-    timed(c, K_NORM, 0, 0, [&] {
-      launch_rmsnorm(c->dtype, c->h, lm_rows, D, m.final_norm, cfg.norm_eps, c->X1, c->act_plane,
-                     gather, head_out ? c->head_w : nullptr, head_out, s);
-    });
     GemmArgs lm = gemm_base(c, m, EPI_STORE, D, c->X1, D, lm_rows);
     lm.w[0] = m.lm_head; lm.seg_rows[0] = cfg.vocab; lm.n_seg = 1; lm.n_virtual = cfg.vocab;
     lm.out_f32 = logits; lm.ld_out = cfg.vocab;
+    if (gather) {   // prefill: normalize the gathered rows explicitly
+      timed(c, K_NORM, 0, 0, [&] {
+        launch_rmsnorm(c->dtype, c->h, lm_rows, D, m.final_norm, cfg.norm_eps, c->X1,
+                       c->act_plane, gather, nullptr, nullptr, s);
+      });
+    } else {
+      normed_input(lm, c->ss_a);
+    }
     gemm(c, lm);
   }
 }
@@ -470,7 +496,7 @@ void do_lookahead(cdsl_ctx* c) {
     const int R = c->B * c->k + (j == 1 ? c->B : 0);
     AttnPass ap;
     ap.rows_per_prompt = c->k + (j == 1 ? 1 : 0);
-    forward(c, c->dft, c->rows_d, R, c->B * c->k, nullptr, c->logits, nullptr, ap);
+    forward(c, c->dft, c->rows_d, R, c->B * c->k, nullptr, c->logits, false, ap);
     RowStatsArgs a{};
     a.logits = c->logits; a.R = c->B * c->k; a.V = c->V; a.k = c->k;
     a.x_out = c->st.x; a.logq_out = c->st.logq; a.out_stride = c->d; a.out_off = j - 1;
@@ -483,12 +509,15 @@ void do_verify(cdsl_ctx* c) {
   timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_verify(c->st, c->rows_v, c->stream); });
   AttnPass ap;
   ap.rows_per_prompt = c->k * (c->d + 1);
-  forward(c, c->tgt, c->rows_v, c->R_v, c->R_v, nullptr, c->logits,
-          c->run.reward_head ? c->st.v_head : nullptr, ap);
+  forward(c, c->tgt, c->rows_v, c->R_v, c->R_v, nullptr, c->logits, c->run.reward_head != 0, ap);
   RowStatsArgs a{};
   a.logits = c->logits; a.R = c->R_v; a.V = c->V; a.k = c->k; a.dp1 = c->d + 1;
   a.next_x = c->st.x; a.amax = c->st.v_amax; a.logp = c->st.v_logp; a.topk = c->st.v_topk;
   a.status = c->st.status;
+  if (c->run.reward_head) {
+    a.ss = c->ss_a; a.hw = c->ss_hw; a.norm_D = c->tcfg.d_model; a.ld_ss = c->R_pad;
+    a.norm_eps = c->tcfg.norm_eps; a.head_out = c->st.v_head;
+  }
   timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
 }
 
@@ -688,14 +717,14 @@ int32_t cdsl_prefill(cdsl_ctx* c, const int32_t* d_prompts, const int32_t* h_pro
     apt.zmap = &zt;
     apd.zmap = &zd;
     apt.n_chunks = apd.n_chunks = (maxpos + attn_chunk()) / attn_chunk();
-    forward(c, c->tgt, c->rows_p, R, nlm, c->lm_gather, c->logits, nullptr, apt);
+    forward(c, c->tgt, c->rows_p, R, nlm, c->lm_gather, c->logits, false, apt);
     if (nlm) {
       RowStatsArgs a{};
       a.logits = c->logits; a.R = nlm; a.V = c->V; a.k = c->k;
       a.topk = st.roots; a.dst = c->lm_dst; a.status = st.status;
       launch_row_stats(a, s);
     }
-    forward(c, c->dft, c->rows_p, R, 0, nullptr, nullptr, nullptr, apd);
+    forward(c, c->dft, c->rows_p, R, 0, nullptr, nullptr, false, apd);
     cudaStreamSynchronize(s);  // host row buffers are reused by the next chunk
     rows.clear(); gather.clear(); dst.clear();
   };

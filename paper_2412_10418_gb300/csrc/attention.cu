@@ -92,12 +92,19 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
     }
     __syncthreads();
   }
-  pdl_wait();                 // q, K/V and the scratch of the previous kernels are ready
-  pdl_launch_dependents();
   const int nq = min(AQB, s_nrows * G - qb * AQB);
-  if (nq <= 0) return;   // no query vector in this block (no block of this group has any)
   int maxnp = 0;
   for (int i = 0; i < nq; ++i) maxnp = max(maxnp, s_np[i]);
+  // Page ids of this chunk: the rows (plan kernel) and the committed page-table entries come
+  // from kernels the launch chain has already completed, so they are read before the wait.
+  if (!tail_chunk && nq > 0 && threadIdx.x < ACH) {
+    const int t = t0 + threadIdx.x;
+    s_page[threadIdx.x] =
+        (t < maxnp) ? a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)] : -1;
+  }
+  pdl_wait();                 // q, K/V and the scratch of the previous kernels are ready
+  pdl_launch_dependents();
+  if (nq <= 0) return;   // no query vector in this block (no block of this group has any)
   const size_t grp = ((size_t)blockIdx.z * gridDim.y + g);
   float* po = a.part_o + (grp * gridDim.x + chunk) * AQB * HD;
   float* pml = a.part_ml + (grp * gridDim.x + chunk) * AQB * 2;
@@ -153,14 +160,8 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
       }
       *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
     }
-    // page ids of this chunk's positions (a chunk spans 64 / page_size pages, at least one)
     const int pmask = (1 << a.kv.page_shift) - 1;
-    if (threadIdx.x < ACH) {
-      const int t = t0 + threadIdx.x;
-      s_page[threadIdx.x] =
-          (t < maxnp) ? a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)] : -1;
-    }
-    __syncthreads();
+    __syncthreads();   // s_page complete
     // every thread first issues all of its K and V loads, then stores them
     constexpr int PER = ACH * (HD / 4) / ATHREADS;   // float4 per thread per matrix
     float4 kr[PER], vr[PER];

@@ -9,6 +9,12 @@
 //   EPI_STORE  : one matrix, fp32 store (logits)
 // Output features are processed in tiles of 128 virtual rows; every pair the epilogue needs
 // (RoPE's (i, i + hd/2), SwiGLU's (gate_j, up_j)) lies inside one tile.
+//
+// RMSNorm is folded into the GEMMs: RMSNorm(h) g W^T = rsqrt(mean(h^2) + eps) * ((h . g) W^T),
+// the row scale factoring out of the dot product. A RESID epilogue therefore also writes the
+// next GEMM's input h . g_next (GEMM-input format) and per 32-feature chunk the partial sums
+// of h^2 (and, for the reward head, of w . g . h); the consuming GEMM's epilogue multiplies by
+// the row scale computed from those partials in a fixed order (deterministic).
 #pragma once
 
 #include "common.cuh"
@@ -42,7 +48,39 @@ struct GemmArgs {
   const RowDesc* rows;     // QKV: per-row position and KV destination
   const float2* rope;      // QKV: [pos][hd/2] (cos, sin)
   int32_t* status;         // device status word (bounded waits report CDSL_ETIMEOUT here)
+  // input normalization: rows are h . g, scale by rsqrt(sum(in_ss[c][r]) / norm_D + eps)
+  const float* in_ss;      // [norm_D / 32][ld_ss] partial sums of squares, or nullptr
+  int32_t norm_D;
+  int32_t ld_ss;           // row stride of the partial-sum arrays (>= R)
+  float norm_eps;
+  // RESID: next GEMM input and its partial sums
+  void* next_x;            // [R, ld_out] GEMM-input format (plane distance act_plane), or nullptr
+  const void* next_g;      // [ld_out] gain of the next RMSNorm (weight dtype)
+  float* out_ss;           // [ld_out / 32][ld_ss]
+  const float* head_w;     // reward head vector [ld_out] (last target layer only), or nullptr
+  float* out_hw;           // [ld_out / 32][ld_ss] partial sums of head_w . g . h
 };
+
+// Row scale rsqrt(mean(h^2) + eps) from the 32-feature partial sums of row r. The partials
+// are summed as four interleaved sequential sums S_q over chunks c = q (mod 4), combined as
+// (S_0 + S_1) + (S_2 + S_3): input_row_scales below takes the same order across four lanes,
+// so every consumer of a row derives the same bits.
+__device__ __forceinline__ float row_scale(const float* ss, int chunks, int ld, int r, int D,
+                                           float eps) {
+  float q[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    q[j] = 0.f;
+    for (int c = j; c < chunks; c += 4) q[j] += ss[(size_t)c * ld + r];
+  }
+  return rsqrtf(((q[0] + q[1]) + (q[2] + q[3])) / (float)D + eps);
+}
+
+// rs[i] = row scale of input row r0 + i for i < n (0 past a.R), computed by `nthr` threads
+// (a multiple of 32, tid = 0 .. nthr-1): lane quads split each row's partials four ways so
+// that all loads of a row are in flight together. The caller synchronizes afterwards.
+__device__ __forceinline__ void input_row_scales(const GemmArgs& a, int r0, int n, float* rs,
+                                                 int tid, int nthr);
 
 // Pointer to virtual row v of the segmented weight matrix, nullptr for padding rows.
 template <typename T>
@@ -64,40 +102,67 @@ __device__ __forceinline__ const T* virtual_row(const GemmArgs& a, int v) {
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }
 
 // Apply the epilogue to a finished fp32 tile: tile[r * ldt + v] holds y for activation row
-// r0 + r and virtual row v0 + v (v in [0, 128)), for r in [0, rt). Run by `nthr` threads
-// (tid = 0 .. nthr-1; all threads of the block by default); the caller synchronizes them
-// before and after.
+// r0 + r and virtual row v0 + v (v in [0, 128)), for r in [0, rt). s_rs[r] is the input row
+// scale of row r0 + r when a.in_ss is set (see input_row_scales). Run by `nthr` threads (a
+// multiple of 32; tid = 0 .. nthr-1; all threads of the block by default), which the caller
+// synchronizes before and after.
 template <typename T>
 __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const float* tile,
-                              int ldt, int tid = -1, int nthr = -1) {
+                              int ldt, const float* s_rs, int tid = -1, int nthr = -1) {
   if (tid < 0) {
     tid = threadIdx.x;
     nthr = blockDim.x;
   }
-  const int n_items = rt * 128;
+  const int n_items = rt * 128;   // a multiple of 32: every warp sees 32 features of one row
   for (int idx = tid; idx < n_items; idx += nthr) {
     const int r = idx >> 7, v = idx & 127;
     const int row = r0 + r;
-    if (row >= a.R) continue;
-    const float y = tile[r * ldt + v];
+    const bool live = row < a.R;
+    float y = tile[r * ldt + v];
+    if (a.in_ss) y *= s_rs[r];
     const int n = v0 + v;
     switch (a.mode) {
       case EPI_STORE:
-        if (n < a.n_virtual) a.out_f32[(size_t)row * a.ld_out + n] = y;
+        if (live && n < a.n_virtual) a.out_f32[(size_t)row * a.ld_out + n] = y;
         break;
-      case EPI_RESID:
-        if (n < a.n_virtual) a.out_f32[(size_t)row * a.ld_out + n] += y;
+      case EPI_RESID: {
+        float hn = 0.f;
+        if (live && n < a.n_virtual) {
+          float* hp = a.out_f32 + (size_t)row * a.ld_out + n;
+          hn = *hp + y;
+          *hp = hn;
+          if (a.next_x)
+            store_act<T>(reinterpret_cast<T*>(a.next_x), a.act_plane, (size_t)row * a.ld_out + n,
+                         hn * to_f32<T>(reinterpret_cast<const T*>(a.next_g)[n]));
+        }
+        if (a.out_ss) {   // warp-uniform: 32 consecutive features of one row
+          const float sq = warp_sum(hn * hn);
+          float hw = 0.f;
+          if (a.head_w) {
+            const float gw = (live && n < a.n_virtual)
+                                 ? a.head_w[n] * to_f32<T>(reinterpret_cast<const T*>(a.next_g)[n])
+                                 : 0.f;
+            hw = warp_sum(gw * hn);
+          }
+          if ((v & 31) == 0 && live && n < a.n_virtual) {
+            a.out_ss[(size_t)(n >> 5) * a.ld_ss + row] = sq;
+            if (a.head_w) a.out_hw[(size_t)(n >> 5) * a.ld_ss + row] = hw;
+          }
+        }
         break;
+      }
       case EPI_SWIGLU: {
-        if (v >= 64) break;
+        if (!live || v >= 64) break;
         const int f = (v0 >> 7) * 64 + v;
         if (f >= a.d_ffn) break;
-        const float u = tile[r * ldt + v + 64];
+        float u = tile[r * ldt + v + 64];
+        if (a.in_ss) u *= s_rs[r];
         store_act<T>(reinterpret_cast<T*>(a.out_act), a.act_plane, (size_t)row * a.ld_act + f,
                      silu_f(y) * u);
         break;
       }
       case EPI_QKV: {
+        if (!live) break;
         const int hd = a.kv.hd, half = hd >> 1;
         const int nq = a.n_heads * hd, nk = a.kv.kvh * hd;
         if (n >= nq + 2 * nk) break;
@@ -106,7 +171,8 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
         const int e = n % hd;  // segments start on head boundaries
         if (n < nq + nk) {     // q or k: rotate-half RoPE with the partner in this tile
           const float2 cs = a.rope[(size_t)rd.pos * half + (e % half)];
-          const float other = (e < half) ? tile[r * ldt + v + half] : tile[r * ldt + v - half];
+          float other = (e < half) ? tile[r * ldt + v + half] : tile[r * ldt + v - half];
+          if (a.in_ss) other *= s_rs[r];
           val = (e < half) ? (y * cs.x - other * cs.y) : (y * cs.x + other * cs.y);
         }
         if (n < nq) {
@@ -128,6 +194,23 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
         break;
       }
     }
+  }
+}
+
+__device__ __forceinline__ void input_row_scales(const GemmArgs& a, int r0, int n, float* rs,
+                                                 int tid, int nthr) {
+  const int chunks = a.norm_D >> 5, items = n * 4;
+  for (int base = tid & ~31; base < items; base += nthr) {   // warp-uniform trip count
+    const int idx = base + (tid & 31), r = idx >> 2, q = idx & 3, row = r0 + r;
+    const bool live = idx < items && row < a.R;
+    float acc = 0.f;
+    if (live) {
+#pragma unroll 8
+      for (int c = q; c < chunks; c += 4) acc += a.in_ss[(size_t)c * a.ld_ss + row];
+    }
+    acc += __shfl_xor_sync(0xffffffffu, acc, 1);   // (S_0 + S_1), (S_2 + S_3)
+    acc += __shfl_xor_sync(0xffffffffu, acc, 2);   // (S_0 + S_1) + (S_2 + S_3)
+    if (idx < items && q == 0) rs[r] = live ? rsqrtf(acc / (float)a.norm_D + a.norm_eps) : 0.f;
   }
 }
 

@@ -19,6 +19,7 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs a) {
   __shared__ float Ws[TK][TV + 1];
   __shared__ float Xs[TK][TR + 1];
   __shared__ float Ys[TR * (TV + 4)];
+  __shared__ float s_rs[TR];
   const int v0 = blockIdx.x * TV;
   const int tid = threadIdx.x;
   const int v = tid & (TV - 1);
@@ -59,8 +60,9 @@ __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs a) {
     }
 #pragma unroll
     for (int i = 0; i < 16; ++i) Ys[(rb + i) * (TV + 4) + v] = acc[i];
+    if (a.in_ss) input_row_scales(a, r0, min(TR, a.R - r0), s_rs, tid, 256);
     __syncthreads();
-    tile_epilogue<T>(a, v0, r0, min(TR, a.R - r0), Ys, TV + 4);
+    tile_epilogue<T>(a, v0, r0, min(TR, a.R - r0), Ys, TV + 4, s_rs);
     __syncthreads();
   }
 }

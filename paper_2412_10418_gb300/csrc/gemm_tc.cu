@@ -69,7 +69,7 @@ __device__ __forceinline__ int unit_start(int c, int U, int C) { return c * U / 
 __device__ __forceinline__ int unit_owner(int u, int U, int C) { return ((u + 1) * C - 1) / U; }
 
 constexpr int kMaxContrib = 256;   // contributors to one tile (bounded on the host)
-constexpr int kMaxSplit = 4;       // target blocks per tile when tiles are few
+constexpr int kMaxSplit = 8;       // target blocks per tile when tiles are few
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_gemm_tc(const __grid_constant__ TcMaps maps, const __grid_constant__ GemmArgs a, TcPlan p,
@@ -82,6 +82,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint32_t tmem_base;
   __shared__ int s_abort, s_last;
   __shared__ int s_slot_off[kMaxContrib];   // reducer: scratch offset (floats) per contributor
+  __shared__ float s_rs[256];                // input row scales (RMSNorm folded into the GEMM)
 
   uint8_t* smem = smem_raw + ((1024 - (tc::smem_u32(smem_raw) & 1023)) & 1023);
   const int NP = p.n_pad, S = p.stages, KBT = p.kb_total;
@@ -230,6 +231,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     int seg = 0;
     int u = u0;
     const int R = min(a.R, NP);
+    if (a.in_ss) {   // once per block, while the first accumulator fills
+      input_row_scales(a, 0, R, s_rs, etid, kEpThreads);
+      tc::named_barrier(1, kEpThreads);
+    }
     while (u < u1) {
       const int t = u / KBT;
       const int seg_end = min(u1, (t + 1) * KBT);
@@ -260,7 +265,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::named_barrier(1, kEpThreads);
         const int rt = max(0, min(rows, R - r0));
         if (whole) {
-          tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, etid, kEpThreads);
+          tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0, etid,
+                                       kEpThreads);
         } else {
           for (int i = etid; i < rt * 128; i += kEpThreads) {
             const int r = i >> 7, v = i & 127;
@@ -312,7 +318,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
             }
             tc::named_barrier(1, kEpThreads);
-            tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, etid, kEpThreads);
+            tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0,
+                                         etid, kEpThreads);
             tc::named_barrier(1, kEpThreads);
           }
           if (etid == 0) tile_cnt[t] = 0;
@@ -328,6 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+size_t g_static_smem = 4096;   // static shared memory of k_gemm_tc (queried at configuration)
 
 }  // namespace
 
@@ -341,15 +349,16 @@ bool tc_supported(const GemmArgs& a) {
   return true;
 }
 
-TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm) {
+TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_split) {
   TcPlan p{};
   p.n_pad = (R + 15) / 16 * 16;
   p.tiles = (n_virtual + 127) / 128;
   p.kb_total = K / 64;
   const size_t stage = 16384 + 256 * (size_t)p.n_pad;
-  // two blocks per SM when three stages fit in half the shared memory, else one; the
+  // two blocks per SM when three stages fit in half the shared memory (228 KB per SM, less
+  // each block's static part and the 1 KB the runtime reserves per block), else one; the
   // epilogue drains 16 activation rows at a time when that frees room for another stage
-  const size_t half = 113 * 1024;
+  const size_t half = 114 * 1024 - g_static_smem - 1024;
   auto fit = [&](size_t budget, int ep) {
     return (int)std::min<size_t>(kMaxStages, (budget - (size_t)ep * kTileLd * 4 - 1024) / stage);
   };
@@ -369,7 +378,7 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm) {
   // at most kMaxSplit blocks share a tile: the fixup then stays cheap next to the streaming
   const long long units = (long long)p.tiles * p.kb_total;
   p.ctas = (int)std::min<long long>(std::min<long long>(units, (long long)per_sm * n_sm),
-                                    (long long)p.tiles * kMaxSplit);
+                                    (long long)p.tiles * (max_split > 0 ? max_split : kMaxSplit));
   p.smem = (size_t)p.stages * stage + tile + 1024;
   return p;
 }
@@ -399,6 +408,9 @@ int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
 }
 
 int configure_gemm_tc() {
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, k_gemm_tc) != cudaSuccess) return -1;
+  g_static_smem = fa.sharedSizeBytes;
   return cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               220 * 1024 + 1024) == cudaSuccess
              ? 0

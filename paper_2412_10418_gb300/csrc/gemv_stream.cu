@@ -128,8 +128,13 @@ __global__ void __launch_bounds__(THREADS) k_gemv(GemmArgs a, int k_split, int n
   }
   __syncthreads();
 
+  __shared__ float s_rs[RM];
+  if (a.in_ss) {
+    input_row_scales(a, 0, min(a.R, RM), s_rs, threadIdx.x, THREADS);
+    __syncthreads();
+  }
   if (n_splits == 1) {
-    tile_epilogue<__nv_bfloat16>(a, v0, 0, min(a.R, RM), tile, TV);
+    tile_epilogue<__nv_bfloat16>(a, v0, 0, min(a.R, RM), tile, TV, s_rs);
     return;
   }
   // split-K: publish this slice's partial tile, the last arriving block reduces and finishes
@@ -152,7 +157,7 @@ __global__ void __launch_bounds__(THREADS) k_gemv(GemmArgs a, int k_split, int n
     tile[i] = s;
   }
   __syncthreads();
-  tile_epilogue<__nv_bfloat16>(a, v0, 0, min(a.R, RM), tile, TV);
+  tile_epilogue<__nv_bfloat16>(a, v0, 0, min(a.R, RM), tile, TV, s_rs);
   if (threadIdx.x == 0) tile_cnt[tile_id] = 0;  // ready for the next launch
 }
 

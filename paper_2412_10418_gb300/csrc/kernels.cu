@@ -3,6 +3,7 @@
 #include <cuda_bf16.h>
 #include <math.h>
 
+#include "gemm.cuh"
 #include "kernels.h"
 
 namespace cdsl {
@@ -38,13 +39,25 @@ __device__ unsigned long long block_max_u64(unsigned long long v, unsigned long 
 }
 
 // ------------------------------------------------------------------------------ embedding
+// h = E[token]; also the first GEMM input x = h . g (GEMM-input format) and the 32-feature
+// partial sums of h^2 from which the consuming GEMM takes the RMSNorm row scale.
 template <typename T>
-__global__ void k_embed(const RowDesc* rows, const T* E, int D, float* h) {
+__global__ void k_embed(const RowDesc* rows, const T* E, int D, float* h, T* x, size_t plane,
+                        const T* g, float* ss, int ld_ss) {
   pdl_wait();
   pdl_launch_dependents();
   const int r = blockIdx.x;
   const T* e = E + (size_t)rows[r].token * D;
-  for (int c = threadIdx.x; c < D; c += blockDim.x) h[(size_t)r * D + c] = to_f32<T>(e[c]);
+  for (int c0 = 0; c0 < D; c0 += blockDim.x) {   // blockDim is a multiple of 32, D of 64
+    const int c = c0 + threadIdx.x;
+    const float v = c < D ? to_f32<T>(e[c]) : 0.f;
+    if (c < D) {
+      h[(size_t)r * D + c] = v;
+      store_act<T>(x, plane, (size_t)r * D + c, v * to_f32<T>(g[c]));
+    }
+    const float sq = warp_sum(v * v);
+    if ((threadIdx.x & 31) == 0 && c < D) ss[(size_t)(c >> 5) * ld_ss + r] = sq;
+  }
 }
 
 // ------------------------------------------------------------------------------ RMSNorm
@@ -153,6 +166,15 @@ __global__ void __launch_bounds__(RS_THREADS) k_row_stats(RowStatsArgs a) {
     return;
   }
   if (a.amax && threadIdx.x == 0) a.amax[r] = amax;
+  if (a.head_out && threadIdx.x < 32) {   // sigmoid(w . g . h * row scale) from the partials
+    float hw = 0.f;
+    for (int c = threadIdx.x; c < (a.norm_D >> 5); c += 32) hw += a.hw[(size_t)c * a.ld_ss + r];
+    hw = warp_sum(hw);
+    if (threadIdx.x == 0) {
+      const float rs = row_scale(a.ss, a.norm_D >> 5, a.ld_ss, r, a.norm_D, a.norm_eps);
+      a.head_out[r] = 1.0f / (1.0f + expf(-hw * rs));
+    }
+  }
   if (a.dp1 > 0 && threadIdx.x == 0) {
     const int j = r % a.dp1, bi = r / a.dp1, d = a.dp1 - 1;
     if (j < d && a.logp) {
@@ -424,8 +446,9 @@ __global__ void k_rope_table(float2* table, int n_pos, int hd, double theta) {
   } while (0)
 
 void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int D, float* h,
-                  cudaStream_t s) {
-  DISPATCH(dtype, launch_pdl(k_embed<T>, dim3(R), dim3(256), 0, s, rows, (const T*)embed, D, h));
+                  void* x, size_t plane, const void* g, float* ss, int ld_ss, cudaStream_t s) {
+  DISPATCH(dtype, launch_pdl(k_embed<T>, dim3(R), dim3(256), 0, s, rows, (const T*)embed, D, h,
+                             (T*)x, plane, (const T*)g, ss, ld_ss));
 }
 
 void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,

@@ -39,8 +39,9 @@ struct StepState {
 };
 
 // elementwise / row kernels (T = float or __nv_bfloat16, the model dtype)
+// h = E[token]; x = h . g in the GEMM-input format; ss = 32-feature partial sums of h^2
 void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int D, float* h,
-                  cudaStream_t s);
+                  void* x, size_t plane, const void* g, float* ss, int ld_ss, cudaStream_t s);
 // out: GEMM-input activations (store_act format, hi/lo planes `plane` elements apart)
 void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
                     void* out, size_t plane, const int32_t* gather, const float* head_w,
@@ -77,6 +78,8 @@ struct RowStatsArgs {
   const int32_t* dst;          // roots: destination row per logits row
   int32_t* x_out; float* logq_out; int32_t out_stride, out_off;  // draft
   int32_t* status;
+  // verify: reward head sigmoid(w . RMSNorm(h)) from the last layer's partial sums
+  const float* ss; const float* hw; int32_t norm_D, ld_ss; float norm_eps; float* head_out;
 };
 void launch_row_stats(const RowStatsArgs& a, cudaStream_t s);
 
@@ -98,7 +101,7 @@ void launch_gemv(const GemmArgs& a, const GemvPlan& p, float* part, int* tile_cn
 struct TcMaps { CUtensorMap w[3]; CUtensorMap xh, xl; };
 struct TcPlan { int tiles, kb_total, ctas, n_pad, stages, ep_rows; size_t smem; };
 bool tc_supported(const GemmArgs& a);
-TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm = 0);
+TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm = 0, int max_split = 0);
 size_t tc_scratch_floats(const TcPlan& p);
 int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                     uint32_t box_inner, uint32_t box_outer);
