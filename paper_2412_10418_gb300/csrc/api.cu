@@ -78,9 +78,6 @@ struct cdsl_ctx {
   int32_t* lm_dst = nullptr;
   float* gemv_part = nullptr;   // split-K partial tiles of the weight-streaming GEMM
   int32_t* gemv_cnt = nullptr;  // per-tile arrival counters
-  float* attn_o = nullptr;      // split-KV attention partials (outputs)
-  float* attn_ml = nullptr;     // split-KV attention partials (max, sum)
-  int32_t* attn_cnt = nullptr;  // per-(query block, head) arrival counters
   int32_t* attn_zmap = nullptr; // prefill: z -> (prompt, query block)
   int attn_zmax = 0, attn_chunks = 0;
   StepState st{};
@@ -150,13 +147,23 @@ int check_run(const cdsl_run_cfg* r, int vocab, std::string* why) {
   if (r->k < 1 || r->k > 16 || r->k > vocab) return bad("k must be in 1..16");
   if (r->d < 1 || r->d > 16) return bad("d must be in 1..16");
   if (r->max_prompt < 1 || r->max_new < 1) return bad("max_prompt and max_new must be >= 1");
-  if ((long long)r->max_prompt + r->max_new > (long long)attn_max_chunks() * attn_chunk())
+  if ((long long)r->max_prompt + r->max_new > (long long)(attn_max_chunks() - 1) * attn_chunk())
     return bad("max_prompt + max_new exceeds the attention limit (4032 positions)");
   if (r->n_keywords < 1 || r->n_keywords > 32) return bad("n_keywords must be in 1..32");
   const int ps = r->page_size ? r->page_size : 64;
   if (ps < 16 || ps > 256 || (ps & (ps - 1))) return bad("page_size must be a power of two in 16..256");
   if (r->max_chunk < 0) return bad("max_chunk must be >= 0");
   return CDSL_OK;
+}
+
+int group_size(const cdsl_model_cfg& m) { return m.n_heads / m.n_kv_heads; }
+int prefix_chunks(const cdsl_run_cfg& r) {
+  return (r.max_prompt + r.max_new + attn_chunk() - 1) / attn_chunk();
+}
+// Most tail-key chunks of any pass: the verify rows of the target, the draft rollout rows.
+int tail_chunks_max(const cdsl_model_cfg& t, const cdsl_model_cfg& dr, const cdsl_run_cfg& r) {
+  return std::max(attn_tail_chunks(r.k * (r.d + 1), group_size(t), r.d + 1, r.d + 1),
+                  attn_tail_chunks(r.k + 1, group_size(dr), 1, r.d));
 }
 
 // Sizes derived from the configurations (shared by cdsl_workspace_size and cdsl_init).
@@ -249,19 +256,12 @@ size_t carve(cdsl_ctx* c, void* base) {
     c->gemv_part = cv.take<float>(part);
     c->gemv_cnt = cv.take<int32_t>(tiles);
   }
-  {  // split-KV attention scratch
+  {  // attention: the prefill's (prompt, query block) map
     const int QB = attn_qblock();
-    const int G = std::max(c->tcfg.n_heads / c->tcfg.n_kv_heads, c->dcfg.n_heads / c->dcfg.n_kv_heads);
-    const int kvh = std::max(c->tcfg.n_kv_heads, c->dcfg.n_kv_heads);
-    const int hd = std::max(c->tcfg.head_dim, c->dcfg.head_dim);
+    const int G = std::max(group_size(c->tcfg), group_size(c->dcfg));
     auto qbs = [&](int rows) { return (rows * G + QB - 1) / QB; };
-    c->attn_zmax = std::max(std::max(B * qbs(k * (d + 1)), B * qbs(k + 1)), qbs(c->R_p) + B);
-    c->attn_chunks = (c->run.max_prompt + c->run.max_new + attn_chunk() - 1) / attn_chunk();
-    const size_t groups = (size_t)c->attn_zmax * kvh;
-    const size_t parts = (size_t)c->attn_chunks + 1;   // prefix chunks + the tail chunk
-    c->attn_o = cv.take<float>(groups * parts * QB * hd);
-    c->attn_ml = cv.take<float>(groups * parts * QB * 2);
-    c->attn_cnt = cv.take<int32_t>(groups);
+    c->attn_zmax = qbs(c->R_p) + B;   // dense passes need no map
+    c->attn_chunks = prefix_chunks(c->run);
     c->attn_zmap = cv.take<int32_t>((size_t)2 * c->attn_zmax);
   }
   StepState& s = c->st;
@@ -401,6 +401,7 @@ struct AttnPass {
   int rows_per_prompt = 0;            // dense: z = b * qb_count + qb
   const std::vector<int32_t>* zmap = nullptr;  // prefill: (b, qb) pairs for this model
   int n_chunks = 0;
+  int n_tchunks = 0;                  // tail-key chunks (attn_tail_chunks)
 };
 
 // One forward pass of a model over R rows described by `rows`; for lm_rows > 0 the final
@@ -418,14 +419,17 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
   at.q = c->qbuf; at.n_heads = H; at.G = H / KVH; at.kv = m.kv; at.rows = rows; at.R = R;
   at.out = c->Xa; at.plane = c->act_plane; at.scale = 1.0f / sqrtf((float)hd);
   at.n_chunks = ap.n_chunks ? ap.n_chunks : c->attn_chunks;
-  at.part_o = c->attn_o; at.part_ml = c->attn_ml; at.cnt = c->attn_cnt;
+  at.n_tchunks = ap.n_tchunks;
+  at.status = c->st.status;
   int n_z;
   if (ap.zmap) {
     n_z = (int)ap.zmap->size() / 2;
     at.zmap = c->attn_zmap;
+    at.qblock = attn_qblock();
     cudaMemcpyAsync(c->attn_zmap, ap.zmap->data(), ap.zmap->size() * 4, cudaMemcpyHostToDevice, s);
   } else {
-    at.qb_count = (ap.rows_per_prompt * at.G + attn_qblock() - 1) / attn_qblock();
+    at.qblock = attn_qblock_for(ap.rows_per_prompt, at.G);
+    at.qb_count = (ap.rows_per_prompt * at.G + at.qblock - 1) / at.qblock;
     n_z = c->B * at.qb_count;
   }
   const int ld_ss = c->R_pad;
@@ -496,6 +500,7 @@ void do_lookahead(cdsl_ctx* c) {
     const int R = c->B * c->k + (j == 1 ? c->B : 0);
     AttnPass ap;
     ap.rows_per_prompt = c->k + (j == 1 ? 1 : 0);
+    ap.n_tchunks = attn_tail_chunks(ap.rows_per_prompt, group_size(c->dcfg), 1, j);
     forward(c, c->dft, c->rows_d, R, c->B * c->k, nullptr, c->logits, false, ap);
     RowStatsArgs a{};
     a.logits = c->logits; a.R = c->B * c->k; a.V = c->V; a.k = c->k;
@@ -509,6 +514,7 @@ void do_verify(cdsl_ctx* c) {
   timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_verify(c->st, c->rows_v, c->stream); });
   AttnPass ap;
   ap.rows_per_prompt = c->k * (c->d + 1);
+  ap.n_tchunks = attn_tail_chunks(ap.rows_per_prompt, group_size(c->tcfg), c->d + 1, c->d + 1);
   forward(c, c->tgt, c->rows_v, c->R_v, c->R_v, nullptr, c->logits, c->run.reward_head != 0, ap);
   RowStatsArgs a{};
   a.logits = c->logits; a.R = c->R_v; a.V = c->V; a.k = c->k; a.dp1 = c->d + 1;
@@ -572,7 +578,12 @@ int validate_all(const cdsl_model_cfg* t, const cdsl_model_cfg* dr, const cdsl_r
   if ((e = check_model(dr, "draft", why))) return e;
   if (t->vocab != dr->vocab) { *why = "target and draft vocabularies differ"; return CDSL_EINVAL; }
   if (t->dtype != dr->dtype) { *why = "target and draft dtypes differ"; return CDSL_EINVAL; }
-  return check_run(r, t->vocab, why);
+  if ((e = check_run(r, t->vocab, why))) return e;
+  if (prefix_chunks(*r) + tail_chunks_max(*t, *dr, *r) > attn_max_chunks()) {
+    *why = "run config: max_prompt + max_new and the beam tails exceed the attention chunks";
+    return CDSL_EINVAL;
+  }
+  return CDSL_OK;
 }
 
 }  // namespace

@@ -1,54 +1,77 @@
 // attention.cu -- attention of every row of a pass over its prompt's shared prefix pages and
 // its own beam tail (decode rows of the draft, the tree-masked verify rows, causal prefill).
 //
-// Prefix sharing: all rows of one prompt read the same prefix K/V. A block owns one prompt,
-// one KV head, one chunk of 64 prefix positions and 32 query vectors (query vector =
-// (row, query head of the GQA group)); it loads the chunk's K and V once into shared memory
-// and scores all its query vectors against them (split-KV, flash-decoding style). One more
-// chunk per query block holds each row's own tail keys (its beam's rows of this pass, causal
-// within the beam). Each query vector's partial result (max score m, sum of exponentials l,
-// unnormalized output o) goes to scratch; the last block of a (prompt, head, query block) to
-// arrive merges the chunks in order (lanes over chunks, all loads in flight) and writes the
-// normalized output in the GEMM-input format. fp32 throughout.
+// Prefix sharing: all rows of one prompt read the same prefix K/V. The keys of a pass are cut
+// into chunks of 64 slots: prefix chunks of 64 consecutive prefix positions, then tail chunks
+// holding the distinct beam tails of a query block's rows (each row masked to its own beam and
+// causal within it). A thread-block cluster of up to 16 blocks owns one prompt, one KV head
+// and one query block of 16 or 32 query vectors (query vector = (row, query head of the GQA
+// group)); block r of the cluster takes chunks r, r + C, ... (one chunk each while the pass
+// has at most 16). For each chunk it loads K and V once into shared memory and scores all its
+// query vectors against them, keeping a running (max m, sum of exponentials l, unnormalized
+// output o) per query vector (split-KV with an online softmax, fp32). The cluster then merges
+// its blocks' partials through distributed shared memory, each block finishing a share of the
+// query vectors, and writes the normalized output in the GEMM-input format. No global scratch,
+// no atomics.
 //
-// Score loop: a warp owns 4 query vectors (broadcast reads), its lanes own keys lane and
-// lane + 32 (rows of 132 floats: conflict-free 128-bit reads). Output loop: lanes own 4 (or 2)
-// consecutive dims of the 4 query vectors, reading P by broadcast and V row-contiguously.
+// Score loop: a warp owns QPW (2 or 4) query vectors (broadcast reads), its lanes own keys lane
+// and lane + 32 (rows of 132 floats: conflict-free 128-bit reads). Output loop: lanes own 4
+// (or 2) consecutive dims of the warp's query vectors, reading P by broadcast and V
+// row-contiguously. All 8 warps have query vectors: a query block is 8 * QPW of them.
 #include <algorithm>
+
+#include <cooperative_groups.h>
 
 #include "kernels.h"
 
 namespace cdsl {
 namespace {
 
-constexpr int ACH = 64;   // prefix positions per block
-constexpr int AQB = 32;   // query vectors per block
+namespace cg = cooperative_groups;
+
+constexpr int ACH = 64;              // key slots per chunk
+constexpr int AQB = 32;              // query vectors per cluster (at most)
+constexpr int MAXP = 64;             // chunks (prefix + tail) of a pass
+constexpr int ACL = 16;              // blocks per cluster (at most)
+constexpr int MAXCB = MAXP / 8;      // chunks per block (at most; clusters have >= 8 blocks
+                                     // whenever a pass has more than 8 chunks)
 constexpr int ATHREADS = 256;
+constexpr int AWARPS = ATHREADS / 32;
+
+int g_max_cluster = 8;               // 16 where non-portable clusters of this kernel fit
 
 template <int HD>
 struct AttnSmem {
   static constexpr int QP = HD + 4;        // padded row pitch of Q and K
-  static constexpr size_t floats = (size_t)AQB * QP + (size_t)ACH * QP + (size_t)ACH * HD + (size_t)ACH * AQB;
+  static constexpr int PP = AQB + 4;       // row pitch of P (4-way store conflicts at most)
+  static constexpr size_t floats = (size_t)AQB * QP + (size_t)ACH * QP + (size_t)ACH * HD + (size_t)ACH * PP;
   static constexpr size_t bytes = floats * sizeof(float);
 };
 
-template <typename T, int HD>
-__global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
+template <typename T, int HD, int QPW>
+__global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   using L = AttnSmem<HD>;
+  constexpr int QB = AWARPS * QPW;              // query vectors of the cluster
   extern __shared__ float4 sm4[];
-  float* qS = reinterpret_cast<float*>(sm4);   // [AQB][QP]  pre-scaled queries
-  float* kS = qS + AQB * L::QP;                 // [ACH][QP]
+  float* qS = reinterpret_cast<float*>(sm4);   // [QB][QP]  pre-scaled queries
+  float* kS = qS + AQB * L::QP;                 // [ACH][QP]; after the chunks: partial o [QB][HD]
   float* vS = kS + ACH * L::QP;                 // [ACH][HD]
-  float* pS = vS + ACH * HD;                    // [ACH][AQB] probabilities
-  __shared__ int s_row[AQB], s_gg[AQB], s_np[AQB];
-  __shared__ int s_wcnt[ATHREADS / 32];
-  __shared__ int s_nrows, s_last;
-  __shared__ float s_m[AQB], s_l[AQB];
-  __shared__ int s_page[ACH];
+  float* pS = vS + ACH * HD;                    // [ACH][PP] probabilities
+  __shared__ int s_row[QB], s_gg[QB], s_np[QB], s_tb[QB], s_nt[QB];
+  __shared__ int s_toff[32], s_tlen[32];        // per query vector: its tail's slot range
+  __shared__ int s_wcnt[AWARPS];
+  __shared__ int s_nrows, s_maxnp;
+  __shared__ float s_pm[QB], s_pl[QB];          // the block's partial (m, l) per query vector
+  __shared__ const float* s_kp[MAXCB * ACH];    // K row of every key slot of the block's chunks
+  __shared__ int s_ktb[MAXCB * ACH];            // tail slots: tail base of the beam,
+  __shared__ uint8_t s_kj[MAXCB * ACH];         //   index in it
 
-  const int chunk = blockIdx.x, g = blockIdx.y;
-  const int n_pchunks = gridDim.x - 1;          // prefix chunks; x == n_pchunks: tail keys
-  const bool tail_chunk = chunk == n_pchunks;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int C = (int)gridDim.x;                 // = cluster size
+  const int cx = (int)blockIdx.x;               // = rank in the cluster
+  const int g = blockIdx.y;
+  const int n_p = a.n_chunks, NC = a.n_chunks + a.n_tchunks;
+  const int nb_chunks = (NC - cx + C - 1) / C;  // this block's chunks cx, cx + C, ...
   int b, qb;
   if (a.zmap) {
     b = a.zmap[2 * blockIdx.z];
@@ -59,15 +82,18 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
   }
   const int G = a.G, H = a.n_heads;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t0 = chunk * ACH;
 
-  // ---- this block's query vectors: rows of prompt b in order, G heads each
-  if (threadIdx.x < AQB) s_row[threadIdx.x] = -1;
+  // ---- this cluster's query vectors: rows of prompt b in order, G heads each. The rows (plan
+  //      kernel), the committed page table and the tail layout come from kernels the launch
+  //      chain has already completed, so everything up to the key slots precedes the wait.
+  if (threadIdx.x < QB) s_row[threadIdx.x] = -1;
+  for (int i = threadIdx.x; i < MAXCB * ACH; i += ATHREADS) s_kp[i] = nullptr;
   if (threadIdx.x == 0) s_nrows = 0;
   __syncthreads();
   for (int base = 0; base < a.R; base += ATHREADS) {
     const int r = base + threadIdx.x;
-    const bool mine = r < a.R && a.rows[r].b == b;
+    RowDesc rd;
+    const bool mine = r < a.R && (rd = a.rows[r]).b == b;
     const unsigned bal = __ballot_sync(0xffffffffu, mine);
     if (lane == 0) s_wcnt[warp] = __popc(bal);
     __syncthreads();
@@ -76,159 +102,219 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
     const int local = off + __popc(bal & ((1u << lane) - 1));
     if (mine) {
       for (int gg = 0; gg < G; ++gg) {
-        const int qi = local * G + gg - qb * AQB;
-        if (qi >= 0 && qi < AQB) {
+        const int qi = local * G + gg - qb * QB;
+        if (qi >= 0 && qi < QB) {
           s_row[qi] = r;
           s_gg[qi] = gg;
-          s_np[qi] = a.rows[r].n_prefix;
+          s_np[qi] = rd.n_prefix;
+          s_tb[qi] = rd.tail_base;
+          s_nt[qi] = rd.n_tail;
         }
       }
     }
     __syncthreads();
     if (threadIdx.x == 0) {
       int tot = 0;
-      for (int w = 0; w < ATHREADS / 32; ++w) tot += s_wcnt[w];
+      for (int w = 0; w < AWARPS; ++w) tot += s_wcnt[w];
       s_nrows += tot;
     }
     __syncthreads();
   }
-  const int nq = min(AQB, s_nrows * G - qb * AQB);
-  int maxnp = 0;
-  for (int i = 0; i < nq; ++i) maxnp = max(maxnp, s_np[i]);
-  // Page ids of this chunk: the rows (plan kernel) and the committed page-table entries come
-  // from kernels the launch chain has already completed, so they are read before the wait.
-  if (!tail_chunk && nq > 0 && threadIdx.x < ACH) {
-    const int t = t0 + threadIdx.x;
-    s_page[threadIdx.x] =
-        (t < maxnp) ? a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)] : -1;
+  const int nq = max(0, min(QB, s_nrows * G - qb * QB));
+  if (warp == 0) {
+    // longest prefix, and the distinct tails (lane = query vector) in order of first
+    // appearance, each as long as its longest row: slot offsets in their concatenation
+    int np = (lane < nq) ? s_np[lane] : 0;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) np = max(np, __shfl_xor_sync(0xffffffffu, np, o));
+    const int tb = (lane < nq) ? s_tb[lane] : -1;
+    const int nt = (lane < nq) ? s_nt[lane] : 0;
+    int len = 0;
+    bool first = nt > 0;
+    for (int j = 0; j < 32; ++j) {
+      const int tbj = __shfl_sync(0xffffffffu, tb, j), ntj = __shfl_sync(0xffffffffu, nt, j);
+      if (tbj == tb && ntj > 0) {
+        len = max(len, ntj);
+        if (j < lane) first = false;
+      }
+    }
+    if (!first) len = 0;
+    int off = len;   // inclusive scan of the lengths over the lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, off, o);
+      if (lane >= o) off += v;
+    }
+    const int total = __shfl_sync(0xffffffffu, off, 31);
+    s_toff[lane] = off - len;
+    s_tlen[lane] = len;
+    if (lane == 0) {
+      s_maxnp = np;
+      if (cx == 0 && total > a.n_tchunks * ACH) set_status(a.status, CDSL_ERANGE);
+    }
   }
-  pdl_wait();                 // q, K/V and the scratch of the previous kernels are ready
+  __syncthreads();
+  const int maxnp = s_maxnp;
+  // key slots of this block's chunks
+  for (int i = 0; i < nb_chunks; ++i) {
+    const int c = cx + i * C;
+    if (c < n_p) {   // prefix positions c*64 .. c*64 + 63 below the longest prefix
+      const int t = c * ACH + (threadIdx.x & (ACH - 1));
+      if (threadIdx.x < ACH && t < maxnp) {
+        const int page = a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)];
+        if (page >= 0)
+          s_kp[i * ACH + threadIdx.x] = a.kv.pool + kv_prefix_offset(a.kv, a.layer, page, 0, g,
+                                                                     t & ((1 << a.kv.page_shift) - 1));
+      }
+    } else if (warp == 0 && lane < nq) {   // tail slots [lo, lo + 64) of the concatenation
+      const int lo = (c - n_p) * ACH, off = s_toff[lane], len = s_tlen[lane], tb = s_tb[lane];
+      for (int e = max(0, lo - off); e < len && off + e < lo + ACH; ++e) {
+        const int sl = i * ACH + off + e - lo;
+        s_kp[sl] = a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, tb + e, g);
+        s_ktb[sl] = tb;
+        s_kj[sl] = (uint8_t)e;
+      }
+    }
+  }
+  __syncthreads();
+  pdl_wait();                 // q and K/V of the previous kernels are ready
   pdl_launch_dependents();
-  if (nq <= 0) return;   // no query vector in this block (no block of this group has any)
-  const size_t grp = ((size_t)blockIdx.z * gridDim.y + g);
-  float* po = a.part_o + (grp * gridDim.x + chunk) * AQB * HD;
-  float* pml = a.part_ml + (grp * gridDim.x + chunk) * AQB * 2;
 
   constexpr int DPL = HD / 32;
-  if (tail_chunk) {
-    // ---- each row's own tail keys (at most 17): lanes over keys for the scores, over dims
-    //      for the output
-    for (int qi = warp; qi < nq; qi += ATHREADS / 32) {
-      const RowDesc rd = a.rows[s_row[qi]];
-      const int nt = min(rd.n_tail, 17);
-      const float* qrow = a.q + (size_t)s_row[qi] * H * HD + (size_t)(g * G + s_gg[qi]) * HD;
-      float sc = -INFINITY;
-      if (lane < nt) {
-        const float* kt = a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, rd.tail_base + lane, g);
-        float d = 0.f;
-#pragma unroll 8
-        for (int e = 0; e < HD; e += 4) {
-          const float4 qv = *reinterpret_cast<const float4*>(qrow + e);
-          const float4 kv = *reinterpret_cast<const float4*>(kt + e);
-          d += qv.x * kv.x + qv.y * kv.y + qv.z * kv.z + qv.w * kv.w;
-        }
-        sc = d * a.scale;
-      }
-      const float m = warp_max(sc);
-      const float pj = (lane < nt) ? expf(sc - m) : 0.f;
-      const float l = warp_sum(pj);
-      float o[DPL];
+  const int q0 = warp * QPW;
+  const bool active = q0 < nq;   // warps without query vectors only help to stage
+  float o[QPW][DPL], m_run[QPW], l_run[QPW];
 #pragma unroll
-      for (int c = 0; c < DPL; ++c) o[c] = 0.f;
-      for (int j = 0; j < nt; ++j) {
-        const float w = __shfl_sync(0xffffffffu, pj, j);
-        const float* vt = a.kv.tail + kv_tail_offset(a.kv, a.layer, 1, rd.tail_base + j, g);
+  for (int i = 0; i < QPW; ++i) {
+    m_run[i] = -INFINITY;
+    l_run[i] = 0.f;
 #pragma unroll
-        for (int c = 0; c < DPL; ++c) o[c] = fmaf(w, vt[DPL * lane + c], o[c]);
-      }
-#pragma unroll
-      for (int c = 0; c < DPL; ++c) po[qi * HD + DPL * lane + c] = o[c];
-      if (lane == 0) {
-        pml[2 * qi] = (nt > 0) ? m : -INFINITY;
-        pml[2 * qi + 1] = l;
-      }
-    }
-  } else if (t0 < maxnp) {
-    // ---- stage Q (scaled), K and V of positions t0 .. t0 + ACH - 1
-    for (int idx = threadIdx.x; idx < AQB * (HD / 4); idx += ATHREADS) {
-      const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (qi < nq) {
-        v = *reinterpret_cast<const float4*>(a.q + (size_t)s_row[qi] * H * HD +
-                                             (size_t)(g * G + s_gg[qi]) * HD + 4 * e4);
-        v.x *= a.scale; v.y *= a.scale; v.z *= a.scale; v.w *= a.scale;
-      }
-      *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
-    }
-    const int pmask = (1 << a.kv.page_shift) - 1;
-    __syncthreads();   // s_page complete
-    // every thread first issues all of its K and V loads, then stores them
+    for (int c = 0; c < DPL; ++c) o[i][c] = 0.f;
+  }
+  bool q_staged = false;
+  for (int i = 0; i < nb_chunks && nq > 0; ++i) {
+    const int c = cx + i * C;
+    const bool tail = c >= n_p;
+    const int t0 = c * ACH;
+    if (!tail && t0 >= maxnp) continue;   // beyond every query vector's prefix
+    // ---- stage K and V of the chunk's 64 slots (and Q the first time), loads in flight
+    //      together
+    constexpr int QPER = QB * (HD / 4) / ATHREADS;
     constexpr int PER = ACH * (HD / 4) / ATHREADS;   // float4 per thread per matrix
-    float4 kr[PER], vr[PER];
+    const size_t v_delta = tail ? (size_t)a.kv.n_tail_slots * a.kv.kvh * HD
+                                : ((size_t)a.kv.kvh << a.kv.page_shift) * HD;
+    float4 qr[QPER], kr[PER], vr[PER];
+    if (!q_staged) {
 #pragma unroll
-    for (int i = 0; i < PER; ++i) {
-      const int idx = threadIdx.x + i * ATHREADS;
-      const int j = idx / (HD / 4), e4 = idx % (HD / 4);
-      const int page = s_page[j];
-      kr[i] = vr[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (page >= 0) {
-        const size_t ko = kv_prefix_offset(a.kv, a.layer, page, 0, g, (t0 + j) & pmask) + 4 * e4;
-        kr[i] = __ldg(reinterpret_cast<const float4*>(a.kv.pool + ko));
-        vr[i] = __ldg(reinterpret_cast<const float4*>(a.kv.pool + ko + ((size_t)a.kv.kvh << a.kv.page_shift) * HD));
+      for (int u = 0; u < QPER; ++u) {
+        const int idx = threadIdx.x + u * ATHREADS;
+        const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
+        qr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (qi < nq)
+          qr[u] = *reinterpret_cast<const float4*>(a.q + (size_t)s_row[qi] * H * HD +
+                                                   (size_t)(g * G + s_gg[qi]) * HD + 4 * e4);
       }
     }
 #pragma unroll
-    for (int i = 0; i < PER; ++i) {
-      const int idx = threadIdx.x + i * ATHREADS;
+    for (int u = 0; u < PER; ++u) {
+      const int idx = threadIdx.x + u * ATHREADS;
       const int j = idx / (HD / 4), e4 = idx % (HD / 4);
-      *reinterpret_cast<float4*>(kS + j * L::QP + 4 * e4) = kr[i];
-      *reinterpret_cast<float4*>(vS + j * HD + 4 * e4) = vr[i];
+      const float* kp = s_kp[i * ACH + j];
+      kr[u] = vr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (kp) {
+        kr[u] = __ldg(reinterpret_cast<const float4*>(kp + 4 * e4));
+        vr[u] = __ldg(reinterpret_cast<const float4*>(kp + v_delta + 4 * e4));
+      }
+    }
+    __syncthreads();   // the previous chunk's readers of kS / vS are done
+    if (!q_staged) {
+#pragma unroll
+      for (int u = 0; u < QPER; ++u) {
+        const int idx = threadIdx.x + u * ATHREADS;
+        const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
+        float4 v = qr[u];
+        v.x *= a.scale; v.y *= a.scale; v.z *= a.scale; v.w *= a.scale;
+        *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
+      }
+      q_staged = true;
+    }
+#pragma unroll
+    for (int u = 0; u < PER; ++u) {
+      const int idx = threadIdx.x + u * ATHREADS;
+      const int j = idx / (HD / 4), e4 = idx % (HD / 4);
+      *reinterpret_cast<float4*>(kS + j * L::QP + 4 * e4) = kr[u];
+      *reinterpret_cast<float4*>(vS + j * HD + 4 * e4) = vr[u];
     }
     __syncthreads();
+    if (!active) continue;
 
-    // ---- scores: warp -> 4 query vectors, lane -> keys lane, lane + 32
-    const int q0 = warp * 4;
-    float s[4][2];
+    // ---- scores: warp -> QPW query vectors, lane -> keys lane, lane + 32
+    float s[QPW][2];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) s[i][0] = s[i][1] = 0.f;
+    for (int q = 0; q < QPW; ++q) s[q][0] = s[q][1] = 0.f;
 #pragma unroll 4
     for (int e = 0; e < HD; e += 4) {
       const float4 k0 = *reinterpret_cast<const float4*>(kS + lane * L::QP + e);
       const float4 k1 = *reinterpret_cast<const float4*>(kS + (lane + 32) * L::QP + e);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float4 qv = *reinterpret_cast<const float4*>(qS + (q0 + i) * L::QP + e);
-        s[i][0] += qv.x * k0.x + qv.y * k0.y + qv.z * k0.z + qv.w * k0.w;
-        s[i][1] += qv.x * k1.x + qv.y * k1.y + qv.z * k1.z + qv.w * k1.w;
+      for (int q = 0; q < QPW; ++q) {
+        const float4 qv = *reinterpret_cast<const float4*>(qS + (q0 + q) * L::QP + e);
+        s[q][0] += qv.x * k0.x + qv.y * k0.y + qv.z * k0.z + qv.w * k0.w;
+        s[q][1] += qv.x * k1.x + qv.y * k1.y + qv.z * k1.z + qv.w * k1.w;
       }
     }
+    // ---- online softmax: running max, rescale of l and o, probabilities of this chunk
+    float p0[QPW], p1[QPW];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int qi = q0 + i;
-      const int np = (qi < nq) ? s_np[qi] : 0;
-      const bool ok0 = t0 + lane < np, ok1 = t0 + lane + 32 < np;
-      const float a0 = ok0 ? s[i][0] : -INFINITY, a1 = ok1 ? s[i][1] : -INFINITY;
-      const float m = warp_max(fmaxf(a0, a1));
-      const float p0 = ok0 ? expf(a0 - m) : 0.f, p1 = ok1 ? expf(a1 - m) : 0.f;
-      const float l = warp_sum(p0 + p1);
-      pS[lane * AQB + qi] = p0;
-      pS[(lane + 32) * AQB + qi] = p1;
-      if (lane == 0) {
-        s_m[qi] = m;
-        s_l[qi] = l;
+    for (int q = 0; q < QPW; ++q) {
+      const int qi = q0 + q;
+      bool ok0, ok1;
+      if (qi >= nq) {
+        ok0 = ok1 = false;
+      } else if (!tail) {         // prefix: positions before the row's prefix length
+        ok0 = t0 + lane < s_np[qi];
+        ok1 = t0 + lane + 32 < s_np[qi];
+      } else {                    // tail: the row's own beam, causal within it
+        const int tb = s_tb[qi], nt = s_nt[qi];
+        const int k0 = i * ACH + lane, k1 = k0 + 32;
+        ok0 = s_kp[k0] && s_ktb[k0] == tb && s_kj[k0] < nt;
+        ok1 = s_kp[k1] && s_ktb[k1] == tb && s_kj[k1] < nt;
       }
+      const float a0 = ok0 ? s[q][0] : -INFINITY, a1 = ok1 ? s[q][1] : -INFINITY;
+      const float m_new = fmaxf(m_run[q], warp_max(fmaxf(a0, a1)));
+      float alpha = 1.f;
+      p0[q] = p1[q] = 0.f;
+      if (m_new > -INFINITY) {
+        alpha = (m_run[q] > -INFINITY) ? expf(m_run[q] - m_new) : 0.f;
+        p0[q] = ok0 ? expf(a0 - m_new) : 0.f;
+        p1[q] = ok1 ? expf(a1 - m_new) : 0.f;
+      }
+      l_run[q] = alpha * l_run[q] + warp_sum(p0[q] + p1[q]);
+      m_run[q] = m_new;
+#pragma unroll
+      for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] *= alpha;
+    }
+    if constexpr (QPW == 4) {
+      *reinterpret_cast<float4*>(pS + lane * L::PP + q0) = make_float4(p0[0], p0[1], p0[2], p0[3]);
+      *reinterpret_cast<float4*>(pS + (lane + 32) * L::PP + q0) =
+          make_float4(p1[0], p1[1], p1[2], p1[3]);
+    } else {
+      *reinterpret_cast<float2*>(pS + lane * L::PP + q0) = make_float2(p0[0], p0[1]);
+      *reinterpret_cast<float2*>(pS + (lane + 32) * L::PP + q0) = make_float2(p1[0], p1[1]);
     }
     __syncwarp();
 
-    // ---- partial output: lane -> dims [DPL*lane, DPL*lane + DPL)
-    float o[4][DPL];
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-#pragma unroll
-      for (int c = 0; c < DPL; ++c) o[i][c] = 0.f;
+    // ---- o += P V: lane -> dims [DPL*lane, DPL*lane + DPL)
 #pragma unroll 4
     for (int t = 0; t < ACH; ++t) {
-      const float4 p4 = *reinterpret_cast<const float4*>(pS + t * AQB + q0);
+      float pp[QPW];
+      if constexpr (QPW == 4) {
+        const float4 p4 = *reinterpret_cast<const float4*>(pS + t * L::PP + q0);
+        pp[0] = p4.x; pp[1] = p4.y; pp[2] = p4.z; pp[3] = p4.w;
+      } else {
+        const float2 p2 = *reinterpret_cast<const float2*>(pS + t * L::PP + q0);
+        pp[0] = p2.x; pp[1] = p2.y;
+      }
       float v[DPL];
       if constexpr (DPL == 4) {
         const float4 v4 = *reinterpret_cast<const float4*>(vS + t * HD + 4 * lane);
@@ -237,117 +323,152 @@ __global__ void __launch_bounds__(ATHREADS) k_attn(AttnArgs a) {
         const float2 v2 = *reinterpret_cast<const float2*>(vS + t * HD + 2 * lane);
         v[0] = v2.x; v[1] = v2.y;
       }
-      const float pp[4] = {p4.x, p4.y, p4.z, p4.w};
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int q = 0; q < QPW; ++q)
 #pragma unroll
-        for (int c = 0; c < DPL; ++c) o[i][c] = fmaf(pp[i], v[c], o[i][c]);
+        for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] = fmaf(pp[q], v[c2], o[q][c2]);
     }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int qi = q0 + i;
-#pragma unroll
-      for (int c = 0; c < DPL; ++c) po[qi * HD + DPL * lane + c] = o[i][c];
-      if (lane == 0) {
-        pml[2 * qi] = s_m[qi];
-        pml[2 * qi + 1] = s_l[qi];
-      }
-    }
+    __syncwarp();   // pS columns of this warp are rewritten by its next chunk
   }
 
-  // ---- last block of this (prompt, head, query block): merge chunks + tail, normalize
-  __threadfence();
+  // ---- the block's partial (m, l, o) per query vector into shared memory (o over kS)
   __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(a.cnt + grp, 1) == (int)gridDim.x - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  // (1) per query vector: max over its chunks and the softmax weight of every chunk
-  constexpr int MAXP = 64;   // prefix chunks + the tail chunk (n_chunks <= 63, checked on the host)
-  float* wS = pS;            // [AQB][MAXP] reuses the probability tile (ACH * AQB floats)
-  static_assert(AQB * MAXP <= ACH * AQB, "merge weights fit in the probability tile");
-  for (int i = threadIdx.x; i < nq * MAXP; i += ATHREADS) {
-    const int qi = i / MAXP, j = i % MAXP;
-    const int ncv = (s_np[qi] + ACH - 1) / ACH;
-    float mc = -INFINITY;
-    if (j <= ncv) {
-      const int cj = j < ncv ? j : n_pchunks;
-      mc = __ldcg(a.part_ml + ((grp * gridDim.x + cj) * AQB + qi) * 2);
-    }
-    wS[i] = mc;
-  }
-  __syncthreads();
-  if (threadIdx.x < nq) {
-    const int qi = threadIdx.x;
-    const int ncv = (s_np[qi] + ACH - 1) / ACH;
-    float m = -INFINITY;
-    for (int j = 0; j <= ncv; ++j) m = fmaxf(m, wS[qi * MAXP + j]);
-    float l = 0.f;
-    for (int j = 0; j <= ncv; ++j) {
-      const float mc = wS[qi * MAXP + j];
-      const int cj = j < ncv ? j : n_pchunks;
-      const float w = (mc > -INFINITY) ? expf(mc - m) : 0.f;
-      l += w * __ldcg(a.part_ml + ((grp * gridDim.x + cj) * AQB + qi) * 2 + 1);
-      wS[qi * MAXP + j] = w;
-    }
-    s_l[qi] = 1.0f / l;
-  }
-  __syncthreads();
-  // (2) outputs: items (query vector, 4 dims), every item's chunk loads in flight together
-  {
-    T* out = reinterpret_cast<T*>(a.out);
-    for (int i = threadIdx.x; i < nq * (HD / 4); i += ATHREADS) {
-      const int qi = i / (HD / 4), e4 = i % (HD / 4);
-      const int ncv = (s_np[qi] + ACH - 1) / ACH;
-      float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-      for (int j = 0; j <= ncv; ++j) {
-        const int cj = j < ncv ? j : n_pchunks;
-        const float w = wS[qi * MAXP + j];
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(
-            a.part_o + ((grp * gridDim.x + cj) * AQB + qi) * HD + 4 * e4));
-        o.x = fmaf(w, v.x, o.x); o.y = fmaf(w, v.y, o.y);
-        o.z = fmaf(w, v.z, o.z); o.w = fmaf(w, v.w, o.w);
+  float* s_po = kS;
+  if (active) {
+#pragma unroll
+    for (int q = 0; q < QPW; ++q) {
+      const int qi = q0 + q;
+      if (qi >= nq) continue;
+#pragma unroll
+      for (int c2 = 0; c2 < DPL; ++c2) s_po[qi * HD + DPL * lane + c2] = o[q][c2];
+      if (lane == 0) {
+        s_pm[qi] = m_run[q];
+        s_pl[qi] = l_run[q];
       }
-      const float inv = s_l[qi];
-      const size_t dst = (size_t)s_row[qi] * H * HD + (size_t)(g * G + s_gg[qi]) * HD + 4 * e4;
-      store_act<T>(out, a.plane, dst + 0, o.x * inv);
-      store_act<T>(out, a.plane, dst + 1, o.y * inv);
-      store_act<T>(out, a.plane, dst + 2, o.z * inv);
-      store_act<T>(out, a.plane, dst + 3, o.w * inv);
     }
   }
-  if (threadIdx.x == 0) a.cnt[grp] = 0;
+  cluster.sync();   // every block's partials are visible to the cluster
+
+  // ---- merge: block cx finishes query vectors cx, cx + C, ... (a warp per query vector),
+  //      reading the C partials through distributed shared memory, 8 blocks at a time
+  for (int qi = cx + warp * C; qi < nq; qi += C * AWARPS) {
+    float mr = -INFINITY, lr = 0.f;
+    if (lane < C) {
+      mr = cluster.map_shared_rank(s_pm, lane)[qi];
+      lr = cluster.map_shared_rank(s_pl, lane)[qi];
+    }
+    const float M = warp_max(mr);
+    const float w = (lane < C && mr > -INFINITY) ? expf(mr - M) : 0.f;
+    const float Lsum = warp_sum(w * lr);
+    float acc[DPL];
+#pragma unroll
+    for (int c2 = 0; c2 < DPL; ++c2) acc[c2] = 0.f;
+    for (int r0 = 0; r0 < C; r0 += 8) {
+      float vv[8][DPL];
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+#pragma unroll
+        for (int c2 = 0; c2 < DPL; ++c2) vv[r][c2] = 0.f;
+        if (r0 + r < C) {
+          const float* src = cluster.map_shared_rank(s_po, r0 + r) + qi * HD + DPL * lane;
+          if constexpr (DPL == 4) {
+            const float4 t4 = *reinterpret_cast<const float4*>(src);
+            vv[r][0] = t4.x; vv[r][1] = t4.y; vv[r][2] = t4.z; vv[r][3] = t4.w;
+          } else {
+            const float2 t2 = *reinterpret_cast<const float2*>(src);
+            vv[r][0] = t2.x; vv[r][1] = t2.y;
+          }
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < 8; ++r) {
+        const float wr = __shfl_sync(0xffffffffu, w, (r0 + r) & 31);
+#pragma unroll
+        for (int c2 = 0; c2 < DPL; ++c2) acc[c2] = fmaf(wr, vv[r][c2], acc[c2]);
+      }
+    }
+    const float inv = Lsum > 0.f ? 1.0f / Lsum : 0.f;
+    T* out = reinterpret_cast<T*>(a.out);
+    const size_t dst = (size_t)s_row[qi] * H * HD + (size_t)(g * G + s_gg[qi]) * HD + DPL * lane;
+#pragma unroll
+    for (int c2 = 0; c2 < DPL; ++c2) store_act<T>(out, a.plane, dst + c2, acc[c2] * inv);
+  }
+  cluster.sync();   // no block leaves while the others may still read its shared memory
 }
 
-template <typename T, int HD>
+template <typename T, int HD, int QPW>
 void launch_t(const AttnArgs& a, int n_z, cudaStream_t s) {
-  dim3 grid(a.n_chunks + 1, a.kv.kvh, n_z);   // + the tail-key chunk
-  launch_pdl(k_attn<T, HD>, grid, dim3(ATHREADS), AttnSmem<HD>::bytes, s, a);
+  const int cl = std::min(g_max_cluster, a.n_chunks + a.n_tchunks);
+  launch_pdl_cluster(k_attn<T, HD, QPW>, dim3(cl, a.kv.kvh, n_z), dim3(ATHREADS),
+                     AttnSmem<HD>::bytes, cl, s, a);
+}
+
+template <typename T, int HD, int QPW>
+int configure_t() {
+  auto k = k_attn<T, HD, QPW>;
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnSmem<HD>::bytes) !=
+      cudaSuccess)
+    return -1;
+  if (cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+    return 1;   // portable clusters only
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(ACL, 1, 1);
+  cfg.blockDim = dim3(ATHREADS);
+  cfg.dynamicSmemBytes = AttnSmem<HD>::bytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = ACL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess || n < 1) {
+    cudaGetLastError();
+    return 1;
+  }
+  return 0;
 }
 
 }  // namespace
 
 int attn_chunk() { return ACH; }
-int attn_max_chunks() { return 63; }
+int attn_max_chunks() { return MAXP; }
 int attn_qblock() { return AQB; }
+int attn_qblock_for(int rows_per_prompt, int G) {
+  return rows_per_prompt * G <= AWARPS * 2 ? AWARPS * 2 : AQB;
+}
+
+int attn_tail_chunks(int rows_per_prompt, int G, int rows_per_tail, int max_tail) {
+  if (max_tail <= 0 || rows_per_prompt <= 0) return 0;
+  // rows met by one query block (it may straddle a row at either end), and the distinct
+  // tails among them when consecutive runs of rows_per_tail rows share one
+  const int rows = std::min(rows_per_prompt, (AQB + G - 1) / G + 1);
+  const int tails = std::min(rows, (rows - 1) / std::max(1, rows_per_tail) + 2);
+  return (tails * max_tail + ACH - 1) / ACH;
+}
 
 int configure_attention() {
-  int e = 0;
-  e |= cudaFuncSetAttribute(k_attn<float, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnSmem<64>::bytes);
-  e |= cudaFuncSetAttribute(k_attn<float, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnSmem<128>::bytes);
-  e |= cudaFuncSetAttribute(k_attn<__nv_bfloat16, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnSmem<64>::bytes);
-  e |= cudaFuncSetAttribute(k_attn<__nv_bfloat16, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnSmem<128>::bytes);
-  return e ? -1 : 0;
+  int worst = 0;
+  for (int r : {configure_t<float, 64, 2>(), configure_t<float, 64, 4>(),
+                configure_t<float, 128, 2>(), configure_t<float, 128, 4>(),
+                configure_t<__nv_bfloat16, 64, 2>(), configure_t<__nv_bfloat16, 64, 4>(),
+                configure_t<__nv_bfloat16, 128, 2>(), configure_t<__nv_bfloat16, 128, 4>()}) {
+    if (r < 0) return -1;
+    worst = std::max(worst, r);
+  }
+  g_max_cluster = worst ? 8 : ACL;
+  return 0;
 }
 
 void launch_attn(int dtype, const AttnArgs& a, int n_z, cudaStream_t s) {
+  const bool q2 = a.qblock <= AWARPS * 2;
   if (dtype == CDSL_DTYPE_BF16) {
-    if (a.kv.hd == 128) launch_t<__nv_bfloat16, 128>(a, n_z, s);
-    else launch_t<__nv_bfloat16, 64>(a, n_z, s);
+    if (a.kv.hd == 128) q2 ? launch_t<__nv_bfloat16, 128, 2>(a, n_z, s) : launch_t<__nv_bfloat16, 128, 4>(a, n_z, s);
+    else q2 ? launch_t<__nv_bfloat16, 64, 2>(a, n_z, s) : launch_t<__nv_bfloat16, 64, 4>(a, n_z, s);
   } else {
-    if (a.kv.hd == 128) launch_t<float, 128>(a, n_z, s);
-    else launch_t<float, 64>(a, n_z, s);
+    if (a.kv.hd == 128) q2 ? launch_t<float, 128, 2>(a, n_z, s) : launch_t<float, 128, 4>(a, n_z, s);
+    else q2 ? launch_t<float, 64, 2>(a, n_z, s) : launch_t<float, 64, 4>(a, n_z, s);
   }
 }
 

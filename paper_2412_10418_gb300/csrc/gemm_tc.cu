@@ -18,6 +18,12 @@
 // the last contributing block of that tile adds the partials in block order (a deterministic
 // sum) and runs the epilogue.
 //
+// Cluster split-K (GEMMs with few tiles): a thread-block cluster of S blocks owns one tile and
+// block r of it the r-th of S even K ranges. Each block drains its partial tile into shared
+// memory; after a cluster barrier every block sums a share of the tile's activation rows over
+// the S partials (in block order, through distributed shared memory) and runs the epilogue on
+// them. No global partials, no atomics.
+//
 // Programmatic dependent launch: weights do not depend on the previous kernel, so the TMA
 // lane issues the first ring's weight loads before griddepcontrol.wait and the activation
 // loads after it; every other dependent access comes after the wait. Every wait on an mbarrier
@@ -26,12 +32,16 @@
 
 #include <algorithm>
 
+#include <cooperative_groups.h>
+
 #include "gemm.cuh"
 #include "kernels.h"
 #include "tc_ptx.cuh"
 
 namespace cdsl {
 namespace {
+
+namespace cg = cooperative_groups;
 
 constexpr int kMaxStages = 8;
 constexpr int kTileLd = 132;     // fp32 epilogue tile row pitch (128 + 4 against bank conflicts)
@@ -92,7 +102,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int c = blockIdx.x, C = gridDim.x;
   const int U = p.tiles * KBT;
-  const int u0 = unit_start(c, U, C), u1 = unit_start(c + 1, U, C);
+  const int SK = p.cluster;   // > 0: cluster split-K, block (tile c / SK, K range c % SK)
+  int u0, u1;
+  if (SK > 0) {
+    const int t = c / SK, r = c % SK;
+    u0 = t * KBT + r * KBT / SK;
+    u1 = t * KBT + (r + 1) * KBT / SK;
+  } else {
+    u0 = unit_start(c, U, C);
+    u1 = unit_start(c + 1, U, C);
+  }
   // hi and lo rows are contiguous in each stage: one MMA with N = 2*NP covers both (the
   // accumulator then holds W.hi in columns [0, NP) and W.lo in [NP, 2NP)); above N = 256 they
   // are two MMAs into one accumulator.
@@ -264,7 +283,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::named_barrier(1, kEpThreads);
         const int rt = max(0, min(rows, R - r0));
-        if (whole) {
+        if (SK > 0 && !whole) {
+          // cluster split-K: the partial stays in tileS (ep_rows == NP: one chunk) until the
+          // cluster reduction below
+        } else if (whole) {
           tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0, etid,
                                        kEpThreads);
         } else {
@@ -277,7 +299,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc::tc_fence_before();
       tc::mbar_arrive(&acce_bar[acc]);   // accumulator drained: the MMA lane may reuse it
-      if (!whole) {
+      if (!whole && SK == 0) {
         const int cf = unit_owner(t * KBT, U, C);
         const int cl = unit_owner((t + 1) * KBT - 1, U, C);
         __threadfence();
@@ -329,6 +351,36 @@ __global__ void __launch_bounds__(kThreads, 1)
       ++seg;
     }
   }
+  if (SK > 0) {
+    // ---- cluster split-K reduction: rank r sums rows [r*R/SK, (r+1)*R/SK) of the SK partial
+    //      tiles in rank order into a free pipeline stage and runs the epilogue on them
+    cg::cluster_group cluster = cg::this_cluster();
+    if (u0 == u1 && warp >= 2)   // empty K range (not planned): contribute zeros
+      for (int i = threadIdx.x - 64; i < NP * kTileLd; i += kEpThreads) tileS[i] = 0.f;
+    __syncthreads();
+    cluster.sync();   // every block's partial tile is complete
+    if (warp >= 2 && !s_abort) {
+      const int etid = threadIdx.x - 64;
+      const int R = min(a.R, NP), r = c % SK, t = c / SK;
+      const int ra = r * R / SK, rb = (r + 1) * R / SK;
+      float* red = reinterpret_cast<float*>(smem);   // stage 0: [rb - ra][kTileLd]
+      for (int i = etid; i < (rb - ra) * 32; i += kEpThreads) {
+        const int off = (ra + (i >> 5)) * kTileLd + (i & 31) * 4;
+        float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q = 0; q < SK; ++q) {
+          const float4 v = *reinterpret_cast<const float4*>(cluster.map_shared_rank(tileS, q) + off);
+          sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
+        }
+        *reinterpret_cast<float4*>(red + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
+      }
+      tc::named_barrier(1, kEpThreads);
+      if (rb > ra)
+        tile_epilogue<__nv_bfloat16>(a, t * 128, ra, rb - ra, red, kTileLd, s_rs + ra, etid,
+                                     kEpThreads);
+    }
+    __syncthreads();
+    cluster.sync();   // no block leaves while another may still read its partial tile
+  }
   tc::tc_fence_before();
   __syncthreads();
   if (warp == 1) tc::tmem_dealloc(tmem, 2 * acc_cols);
@@ -349,7 +401,8 @@ bool tc_supported(const GemmArgs& a) {
   return true;
 }
 
-TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_split) {
+TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_split,
+               int cluster) {
   TcPlan p{};
   p.n_pad = (R + 15) / 16 * 16;
   p.tiles = (n_virtual + 127) / 128;
@@ -374,16 +427,28 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   }
   p.ep_rows = fit(budget, 16) > fit(budget, ep_big) ? 16 : ep_big;
   p.stages = fit(budget, p.ep_rows);
-  const size_t tile = (size_t)p.ep_rows * kTileLd * 4;
   // at most kMaxSplit blocks share a tile: the fixup then stays cheap next to the streaming
   const long long units = (long long)p.tiles * p.kb_total;
   p.ctas = (int)std::min<long long>(std::min<long long>(units, (long long)per_sm * n_sm),
                                     (long long)p.tiles * (max_split > 0 ? max_split : kMaxSplit));
-  p.smem = (size_t)p.stages * stage + tile + 1024;
+  // few tiles: a cluster of S blocks per tile (all tiles resident at once, S <= 8 portable)
+  const int cap = per_sm * n_sm;
+  int S = cluster;
+  if (S < 0) S = (p.n_pad <= kEpRowsMax && 2 * p.tiles <= cap) ? std::min(8, cap / p.tiles) : 0;
+  S = std::min(S, p.kb_total);
+  if (S >= 2 && p.n_pad <= kEpRowsMax) {
+    p.cluster = S;
+    p.ctas = p.tiles * S;
+    p.ep_rows = p.n_pad;   // the whole partial tile stays in shared memory
+    p.stages = fit(budget, p.ep_rows);
+  }
+  p.smem = (size_t)p.stages * stage + (size_t)p.ep_rows * kTileLd * 4 + 1024;
   return p;
 }
 
-size_t tc_scratch_floats(const TcPlan& p) { return (size_t)p.ctas * 2 * p.n_pad * 128; }
+size_t tc_scratch_floats(const TcPlan& p) {
+  return p.cluster ? 0 : (size_t)p.ctas * 2 * p.n_pad * 128;
+}
 
 int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                     uint32_t box_inner, uint32_t box_outer) {
@@ -419,7 +484,11 @@ int configure_gemm_tc() {
 
 void launch_gemm_tc(const TcMaps& maps, const GemmArgs& a, const TcPlan& p, float* part,
                     int* tile_cnt, cudaStream_t s) {
-  launch_pdl(k_gemm_tc, dim3(p.ctas), dim3(kThreads), p.smem, s, maps, a, p, part, tile_cnt);
+  if (p.cluster)
+    launch_pdl_cluster(k_gemm_tc, dim3(p.ctas), dim3(kThreads), p.smem, p.cluster, s, maps, a, p,
+                       part, tile_cnt);
+  else
+    launch_pdl(k_gemm_tc, dim3(p.ctas), dim3(kThreads), p.smem, s, maps, a, p, part, tile_cnt);
 }
 
 }  // namespace cdsl

@@ -46,23 +46,29 @@ void launch_embed(int dtype, const RowDesc* rows, int R, const void* embed, int 
 void launch_rmsnorm(int dtype, const float* h, int R, int D, const void* gain, float eps,
                     void* out, size_t plane, const int32_t* gather, const float* head_w,
                     float* head_out, cudaStream_t s);
-// Attention of a pass (attention.cu). Blocks: (prefix chunk of attn_chunk() positions or the
-// tail-key chunk, kv head, z) with z -> (prompt, query block of attn_qblock() query vectors)
-// either dense (b = z / qb_count) or from zmap[2z], zmap[2z+1]. Scratch: part_o
-// [n_z][kvh][n_chunks + 1][qblock][hd], part_ml [n_z][kvh][n_chunks + 1][qblock][2],
-// cnt [n_z][kvh] (zero between launches).
+// Attention of a pass (attention.cu). Chunks 0 .. n_chunks-1 hold attn_chunk() prefix
+// positions each, the n_tchunks after them the query blocks' beam tails (n_chunks + n_tchunks
+// <= attn_max_chunks()). Grid: (cluster of up to 16 blocks over the chunks, kv head, z) with
+// z -> (prompt, query block of `qblock` query vectors: attn_qblock_for(), or attn_qblock()
+// with a zmap) either dense (b = z / qb_count) or from zmap[2z], zmap[2z+1]. More tail keys
+// than the tail chunks hold latch CDSL_ERANGE in *status.
 struct AttnArgs {
   const float* q; int32_t n_heads, G;
   KvStore kv; int32_t layer;
   const RowDesc* rows; int32_t R;
   void* out; size_t plane; float scale;
-  int32_t n_chunks, qb_count;
+  int32_t n_chunks, n_tchunks, qb_count, qblock;
   const int32_t* zmap;
-  float* part_o; float* part_ml; int32_t* cnt;
+  int32_t* status;
 };
 int attn_chunk();
 int attn_max_chunks();
 int attn_qblock();
+// Query vectors per block of a dense pass with rows_per_prompt rows per prompt, GQA group G.
+int attn_qblock_for(int rows_per_prompt, int G);
+// Tail chunks a pass needs: rows_per_prompt rows per prompt, GQA group G, consecutive runs of
+// rows_per_tail rows sharing one beam tail, tails of at most max_tail keys.
+int attn_tail_chunks(int rows_per_prompt, int G, int rows_per_tail, int max_tail);
 int configure_attention();
 void launch_attn(int dtype, const AttnArgs& a, int n_z, cudaStream_t s);
 // Row statistics of logits rows: argmax (lower id on ties), log-sum-exp, top-k, log p.
@@ -99,9 +105,14 @@ void launch_gemv(const GemmArgs& a, const GemvPlan& p, float* part, int* tile_cn
 // Scratch: part [ctas][2][n_pad][128] floats (tc_scratch_floats), one arrival counter per
 // tile (zero between launches). Launched with programmatic dependent launch allowed.
 struct TcMaps { CUtensorMap w[3]; CUtensorMap xh, xl; };
-struct TcPlan { int tiles, kb_total, ctas, n_pad, stages, ep_rows; size_t smem; };
+// cluster > 0: cluster split-K with that many blocks per tile (ctas = tiles * cluster); 0:
+// persistent stream-K over ctas blocks.
+struct TcPlan { int tiles, kb_total, ctas, n_pad, stages, ep_rows, cluster; size_t smem; };
 bool tc_supported(const GemmArgs& a);
-TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm = 0, int max_split = 0);
+// cluster: -1 chooses (split-K clusters when every tile fits at once with >= 2 blocks), 0
+// stream-K, > 0 that cluster size.
+TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm = 0, int max_split = 0,
+               int cluster = -1);
 size_t tc_scratch_floats(const TcPlan& p);
 int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
                     uint32_t box_inner, uint32_t box_outer);

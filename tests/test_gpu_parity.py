@@ -74,8 +74,10 @@ def test_ragged_batch_small_pages():
     tokens_match(eng, states)
 
 
-@pytest.mark.parametrize("k,d", [(1, 1), (2, 3), (16, 2)])
+@pytest.mark.parametrize("k,d", [(1, 1), (2, 3), (16, 2), (8, 12)])
 def test_beam_and_lookahead_extremes(k, d):
+    """(8, 12) with one query head per KV head: the draft rows' beam tails (up to 8 x 12 keys
+    per query block) span two tail-key chunks of the attention."""
     wl = synth.scaled(synth.TINY, k=k, d=d, max_new=7)
     s = make_setup(wl)
     eng, states, rep, adopted, n = run_parity(s, steps=10, tol=TOL32, tol_r=TOL32)
