@@ -388,6 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 size_t g_static_smem = 4096;   // static shared memory of k_gemm_tc (queried at configuration)
+int g_max_cluster = 8;         // 16 where non-portable clusters of k_gemm_tc are allowed
 
 }  // namespace
 
@@ -431,11 +432,13 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   const long long units = (long long)p.tiles * p.kb_total;
   p.ctas = (int)std::min<long long>(std::min<long long>(units, (long long)per_sm * n_sm),
                                     (long long)p.tiles * (max_split > 0 ? max_split : kMaxSplit));
-  // few tiles: a cluster of S blocks per tile (all tiles resident at once, S <= 8 portable)
-  const int cap = per_sm * n_sm;
+  // few tiles: a cluster of S <= 8 blocks per tile, all tiles resident at once. Clusters are
+  // placed whole within a GPC; on 152 SMs at two blocks each, grids of clusters past ~87 % of
+  // the block slots no longer fit in one wave (measured), hence the cap.
+  const int cap = per_sm * n_sm * 87 / 100;
   int S = cluster;
   if (S < 0) S = (p.n_pad <= kEpRowsMax && 2 * p.tiles <= cap) ? std::min(8, cap / p.tiles) : 0;
-  S = std::min(S, p.kb_total);
+  S = std::min(std::min(S, p.kb_total), g_max_cluster);
   if (S >= 2 && p.n_pad <= kEpRowsMax) {
     p.cluster = S;
     p.ctas = p.tiles * S;
@@ -476,6 +479,11 @@ int configure_gemm_tc() {
   cudaFuncAttributes fa;
   if (cudaFuncGetAttributes(&fa, k_gemm_tc) != cudaSuccess) return -1;
   g_static_smem = fa.sharedSizeBytes;
+  g_max_cluster =
+      cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess
+          ? 16
+          : 8;
+  cudaGetLastError();
   return cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               220 * 1024 + 1024) == cudaSuccess
              ? 0
