@@ -32,16 +32,12 @@
 
 #include <algorithm>
 
-#include <cooperative_groups.h>
-
 #include "gemm.cuh"
 #include "kernels.h"
 #include "tc_ptx.cuh"
 
 namespace cdsl {
 namespace {
-
-namespace cg = cooperative_groups;
 
 constexpr int kMaxStages = 8;
 constexpr int kTileLd = 132;     // fp32 epilogue tile row pitch (128 + 4 against bank conflicts)
@@ -118,7 +114,31 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool fused = 2 * NP <= 256;
   const uint32_t acc_cols = tmem_cols_for(fused ? 2 * NP : NP);
 
+  // TMA producer state (thread 0): unit u0 + i is (t_cur, kb_cur) for the next i to issue
+  const int n_units = u1 - u0;
+  const int pre = min(S, n_units);
+  int t_cur = u0 / KBT, kb_cur = u0 % KBT;
+  uint64_t pol = 0;
+  auto load_w = [&](int i, int t, int kb) {
+    int m0, y0, m1, y1;
+    half_source(a, t * 128, &m0, &y0);
+    half_source(a, t * 128 + 64, &m1, &y1);
+    uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
+    tc::tma_load_2d_hint(st, &maps.w[m0], kb * 64, y0, &full_bar[i % S], pol);
+    tc::tma_load_2d_hint(st + 8192, &maps.w[m1], kb * 64, y1, &full_bar[i % S], pol);
+  };
+  auto load_x = [&](int i, int kb) {
+    uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
+    for (int j = 0; j < NP / 16; ++j) {
+      tc::tma_load_2d(st + 16384 + j * 2048, &maps.xh, kb * 64, j * 16, &full_bar[i % S]);
+      tc::tma_load_2d(st + 16384 + NP * 128 + j * 2048, &maps.xl, kb * 64, j * 16,
+                      &full_bar[i % S]);
+    }
+  };
   if (threadIdx.x == 0) {
+    for (int m = 0; m < 3; ++m) tc::tma_prefetch_map(&maps.w[m]);
+    tc::tma_prefetch_map(&maps.xh);
+    tc::tma_prefetch_map(&maps.xl);
     for (int s = 0; s < S; ++s) {
       tc::mbar_init(&full_bar[s], 1);
       tc::mbar_init(&empty_bar[s], 1);
@@ -129,6 +149,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     s_abort = 0;
     tc::fence_mbar_init();
+    tc::fence_proxy_async();
+    // the first ring's weights do not depend on the previous kernel: issue them while warp 1
+    // allocates TMEM
+    pol = tc::policy_evict_first();
+    for (int i = 0; i < pre; ++i) {
+      tc::mbar_expect_tx(&full_bar[i], stage_bytes);
+      load_w(i, t_cur, kb_cur);
+      if (++kb_cur == KBT) { kb_cur = 0; ++t_cur; }
+    }
   }
   if (warp == 1) tc::tmem_alloc(&tmem_base, 2 * acc_cols);
   tc::tc_fence_before();
@@ -140,34 +169,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer
-      const uint64_t pol = tc::policy_evict_first();
-      const int n = (int)(u1 - u0);
-      const int pre = min(S, n);
       bool aborted = false;
       int issued = 0;
-      int t_cur = u0 / KBT, kb_cur = u0 % KBT;   // unit u0 + i, advanced incrementally
-      auto load_w = [&](int i, int t, int kb) {
-        int m0, y0, m1, y1;
-        half_source(a, t * 128, &m0, &y0);
-        half_source(a, t * 128 + 64, &m1, &y1);
-        uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
-        tc::tma_load_2d_hint(st, &maps.w[m0], kb * 64, y0, &full_bar[i % S], pol);
-        tc::tma_load_2d_hint(st + 8192, &maps.w[m1], kb * 64, y1, &full_bar[i % S], pol);
-      };
-      auto load_x = [&](int i, int kb) {
-        uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
-        for (int j = 0; j < NP / 16; ++j) {
-          tc::tma_load_2d(st + 16384 + j * 2048, &maps.xh, kb * 64, j * 16, &full_bar[i % S]);
-          tc::tma_load_2d(st + 16384 + NP * 128 + j * 2048, &maps.xl, kb * 64, j * 16,
-                          &full_bar[i % S]);
-        }
-      };
-      // the first ring's weights do not depend on the previous kernel
-      for (int i = 0; i < pre; ++i) {
-        tc::mbar_expect_tx(&full_bar[i], stage_bytes);
-        load_w(i, t_cur, kb_cur);
-        if (++kb_cur == KBT) { kb_cur = 0; ++t_cur; }
-      }
       pdl_wait();
       {
         int kb = u0 % KBT;
@@ -177,7 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       issued = pre;
-      for (int i = pre; i < n; ++i) {
+      for (int i = pre; i < n_units; ++i) {
         const int s = i % S, use = i / S;
         if (!tc::mbar_wait(&empty_bar[s], (use - 1) & 1, a.status)) {
           aborted = true;
@@ -283,9 +286,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::named_barrier(1, kEpThreads);
         const int rt = max(0, min(rows, R - r0));
-        if (SK > 0 && !whole) {
+        if (SK > 0) {
           // cluster split-K: the partial stays in tileS (ep_rows == NP: one chunk) until the
-          // cluster reduction below
+          // cluster reduction at the end
         } else if (whole) {
           tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0, etid,
                                        kEpThreads);
@@ -353,22 +356,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (SK > 0) {
     // ---- cluster split-K reduction: rank r sums rows [r*R/SK, (r+1)*R/SK) of the SK partial
-    //      tiles in rank order into a free pipeline stage and runs the epilogue on them
-    cg::cluster_group cluster = cg::this_cluster();
-    if (u0 == u1 && warp >= 2)   // empty K range (not planned): contribute zeros
-      for (int i = threadIdx.x - 64; i < NP * kTileLd; i += kEpThreads) tileS[i] = 0.f;
-    __syncthreads();
-    cluster.sync();   // every block's partial tile is complete
+    //      tiles in rank order (distributed shared memory) into a free pipeline stage and runs
+    //      the epilogue on them
+    tc::cluster_arrive();               // this block's partial tile is complete (release)
+    tc::cluster_wait();                 // every block's is (acquire)
     if (warp >= 2 && !s_abort) {
       const int etid = threadIdx.x - 64;
       const int R = min(a.R, NP), r = c % SK, t = c / SK;
       const int ra = r * R / SK, rb = (r + 1) * R / SK;
-      float* red = reinterpret_cast<float*>(smem);   // stage 0: [rb - ra][kTileLd]
+      float* red = reinterpret_cast<float*>(smem);   // stage 0 (idle): [rb - ra][kTileLd]
+      const uint32_t tile_s = tc::smem_u32(tileS);
       for (int i = etid; i < (rb - ra) * 32; i += kEpThreads) {
-        const int off = (ra + (i >> 5)) * kTileLd + (i & 31) * 4;
+        const uint32_t off = ((ra + (i >> 5)) * kTileLd + (i & 31) * 4) * 4;
         float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int q = 0; q < SK; ++q) {
-          const float4 v = *reinterpret_cast<const float4*>(cluster.map_shared_rank(tileS, q) + off);
+          const float4 v = tc::ld_cluster_f32x4(tc::map_cluster_rank(tile_s + off, q));
           sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
         }
         *reinterpret_cast<float4*>(red + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
@@ -378,8 +380,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         tile_epilogue<__nv_bfloat16>(a, t * 128, ra, rb - ra, red, kTileLd, s_rs + ra, etid,
                                      kEpThreads);
     }
-    __syncthreads();
-    cluster.sync();   // no block leaves while another may still read its partial tile
+    tc::cluster_arrive_relaxed();       // this block has read the others' tiles
+    tc::cluster_wait();                 // no block leaves while its tile may still be read
   }
   tc::tc_fence_before();
   __syncthreads();

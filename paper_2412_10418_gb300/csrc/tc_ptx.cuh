@@ -31,6 +31,10 @@ __device__ __forceinline__ void mbar_init(uint64_t* m, uint32_t count) {
 __device__ __forceinline__ void fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
+// Order this thread's generic-proxy shared-memory writes before later async-proxy (TMA) use.
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 __device__ __forceinline__ void mbar_expect_tx(uint64_t* m, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(m)), "r"(bytes)
                : "memory");
@@ -65,6 +69,35 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* m, uint32_t parity, int32_t*
     }
   }
   return true;
+}
+
+// ------------------------------------------------------------------------------ cluster
+// Split cluster barrier: every thread of every block of the cluster arrives, then waits for
+// the phase. A relaxed arrive orders nothing; the default arrive releases this thread's prior
+// memory accesses and the wait acquires the others' (shared::cluster included).
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait;" ::: "memory");
+}
+// Shared-memory address of the same variable in block `rank` of this cluster (for
+// ld/st.shared::cluster).
+__device__ __forceinline__ uint32_t map_cluster_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float4 ld_cluster_f32x4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
 }
 
 // ------------------------------------------------------------------------------ TMA
