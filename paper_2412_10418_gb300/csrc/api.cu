@@ -309,7 +309,7 @@ double gemm_bytes(const cdsl_ctx* c, const GemmArgs& a, double* flops) {
   double out = 0;
   switch (a.mode) {
     case EPI_STORE: out = 4.0 * a.R * rows; break;
-    case EPI_RESID: out = 8.0 * a.R * rows; break;
+    case EPI_RESID: out = (a.next_x ? 12.0 : 8.0) * a.R * rows; break;   // h r/w (+ next input)
     case EPI_SWIGLU: out = 4.0 * a.R * a.d_ffn; break;
     case EPI_QKV: out = 4.0 * a.R * rows; break;
   }
