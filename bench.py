@@ -38,6 +38,11 @@ def parse():
     ap.add_argument("--workload", default="7b-bf16")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--acceptance", choices=["hard", "speculative"], default="hard",
+                    help="validation of the lookaheads by M_p (Sec. 3.2.2)")
+    ap.add_argument("--decoder", choices=["cdsl", "cdlh"], default="cdsl",
+                    help="cdlh: the lookaheads come from M_p itself and no lookahead is ever "
+                         "accepted (Alg. 2 CDLH on the same kernels)")
     ap.add_argument("--oracle-layers", type=int, default=2,
                     help="target layers the oracle sample runs (scaled to the full depth)")
     return ap.parse_args()
@@ -134,20 +139,27 @@ class ClockSampler:
 
 # ------------------------------------------------------------------------------ GPU arm
 
-def build_engine(wl, device):
+def build_engine(wl, device, acceptance="hard", decoder="cdsl"):
+    """The CDSL-k engine of a workload. decoder "cdlh": M_p drafts its own lookaheads and the
+    reward threshold is above any reward (S1 never holds), so every step emits the one token
+    of Alg. 2's CDLH (the step still runs its verify pass, which scores the beams)."""
     import torch
     import synth
     import paper_2412_10418_gb300 as cdsl
 
     tw = synth.model_weights(wl, "target", device=device)
-    dw = synth.model_weights(wl, "draft", device=device)
+    cdlh = decoder == "cdlh"
+    dw = tw if cdlh else synth.model_weights(wl, "draft", device=device)
+    dshape = wl.target if cdlh else wl.draft
     head = torch.from_numpy(synth.reward_head(wl)).to(device) if wl.reward_head else None
-    eng = cdsl.Engine(wl.target, wl.draft, wl.dtype,
+    eng = cdsl.Engine(wl.target, dshape, wl.dtype,
                       [tw[n] for n, _ in wl.target.weight_specs()],
-                      [dw[n] for n, _ in wl.draft.weight_specs()],
+                      [dw[n] for n, _ in dshape.weight_specs()],
                       batch=wl.batch, k=wl.k, d=wl.d, max_prompt=wl.prompt_len,
-                      max_new=wl.max_new, n_keywords=wl.n_keywords, a_t=wl.a_t, r_t=wl.r_t,
-                      reward_head=head, device=device)
+                      max_new=wl.max_new, n_keywords=wl.n_keywords, a_t=wl.a_t,
+                      r_t=2.0 if cdlh else wl.r_t, reward_head=head,
+                      acceptance=cdsl.ACCEPT_SPECULATIVE if acceptance == "speculative"
+                      else cdsl.ACCEPT_HARD, seed=1, device=device)
     return eng, tw, dw
 
 
@@ -220,12 +232,13 @@ def kernel_timing(eng, wl, n_steps):
 
 
 def e2e_run(eng, wl, n_steps):
-    """tokens/s through the public API with host buffers: pinned prompts and keywords are
-    copied in, the prompts prefilled, then every step's emitted tokens are read back."""
+    """tokens/s through the public API with host buffers, for whole generations: pinned
+    prompts and keywords are copied in, the prompts prefilled, then steps run until every
+    prompt has its l_m tokens, each step's emitted tokens read back to the host."""
     import torch
     import synth
     import paper_2412_10418_gb300 as cdsl
-    n_steps = min(n_steps, max(1, wl.max_new // (wl.d + 1)))
+    n_steps = wl.max_new     # at least one token per step per live prompt
     hp = torch.from_numpy(synth.prompts(wl)).pin_memory()
     hk = torch.from_numpy(synth.keywords(wl)).pin_memory()
     out_tok = torch.empty((wl.batch, wl.d + 1), dtype=torch.int32).pin_memory()
@@ -239,6 +252,7 @@ def e2e_run(eng, wl, n_steps):
         dk.copy_(hk, non_blocking=True)
     cdsl.cdsl_prefill(eng.ctx, dp, [wl.prompt_len] * wl.batch, dk)
     tokens = 0
+    done = 0
     for _ in range(n_steps):
         eng.step()
         with torch.cuda.stream(eng.stream):
@@ -246,7 +260,11 @@ def e2e_run(eng, wl, n_steps):
             out_n.copy_(eng.n_emitted, non_blocking=True)
         eng.stream.synchronize()
         tokens += int(out_n.sum())
+        done += 1
+        if tokens >= wl.batch * wl.max_new:
+            break
     dt = time.perf_counter() - t0
+    n_steps = done
     h2d = (hp.numel() + hk.numel()) * 4 / n_steps
     d2h = (out_tok.numel() + out_n.numel()) * 4
     return tokens / dt, h2d, d2h, n_steps
@@ -340,7 +358,7 @@ def gpu_main(args):
     if world > 1:
         dist.barrier()
     wl = workload(args.workload)
-    eng, tw, dw = build_engine(wl, device)
+    eng, tw, dw = build_engine(wl, device, args.acceptance, args.decoder)
 
     if world > 1:
         dist.barrier()
@@ -385,20 +403,24 @@ def gpu_main(args):
             ev = float(t[0])
         e2e = {"value": round(ev, 3), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d, 1),
                "d2h_bytes_per_step": d2h,
-               "note": f"pinned prompts+keywords in, prefill, then {n_e2e} cdsl_step calls each "
+               "note": f"whole generations: pinned prompts+keywords in, prefill, then {n_e2e} "
+                       "cdsl_step calls (until every prompt has max_new tokens), each "
                        "followed by a read of the emitted tokens"}
     out = None
     if rank == 0:
         tokens_per_step = tokens / (args.steps * max(1, world)) / wl.batch
         cpu = None
-        if not args.no_cpu_baseline and world == 1:
+        if not args.no_cpu_baseline and world == 1 and args.decoder == "cdsl":
             cpu = cpu_baseline(wl, tw, dw, tokens_per_step, args.oracle_layers)
         out = {
             "metric": METRIC, "value": round(value, 3), "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": dict(config_of(wl), parallelism=f"replicas{world}"),
+            "config": dict(config_of(wl), parallelism=f"replicas{world}",
+                           acceptance=args.acceptance, decoder=args.decoder,
+                           **({"draft": "= target (CDLH)", "r_t": None}
+                              if args.decoder == "cdlh" else {})),
             "verify_us": round(verify_us, 1),
             "verify_gbs": round(verify_bytes / (verify_us * 1e-6) / 1e9, 1),
             "tokens_per_step": round(tokens_per_step, 3),

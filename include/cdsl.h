@@ -87,8 +87,17 @@ typedef struct cdsl_run_cfg {
   float r_t;            /* reward threshold */
   int32_t reward_head;  /* 0: R = coverage; 1: R = 0.5 coverage + 0.5 sigmoid(w . h_last) */
   int32_t page_size;    /* KV page size in tokens (power of two, 16..256); 0 = 64 */
-  int32_t max_chunk;    /* rows per prefill forward pass; 0 = 256 */
-  int32_t reserved;
+  int32_t max_chunk;    /* rows per prefill forward pass; 0 = 64 */
+  /* Validation of the lookahead by M_p (Sec. 3.2.2):
+   *   0: hard rejection: x_j is accepted while argmax p_j == x_j;
+   *   1: speculative sampling: x_j is accepted while u_j <= min(1, p_j(x_j) / q_j(x_j)),
+   *      tested as log(u_j) <= log p_j(x_j) - log q_j(x_j) in float32. The rejected position's
+   *      resampled token is never emitted, so only the count n_b is used.
+   * u_j = (SplitMix64 output number c of the generator seeded with `seed`) >> 40, times 2^-24,
+   * where c = ((step * batch + b) * k + beam) * d + (j - 1) and step counts the completed
+   * steps of the context (SplitMix64: Steele, Lea, Flood, OOPSLA 2014). */
+  int32_t acceptance;
+  uint32_t seed;
 } cdsl_run_cfg;
 
 typedef struct cdsl_ctx cdsl_ctx;

@@ -13,6 +13,8 @@ prompt):
   2. x_{b,1..d} = greedy rollout of M_q from pfx + c_b                 (Sec. 3.2.1, Alg. 1)
   3. p_{b,1..d+1} = M_p(pfx + c_b + x_{b,<j}), j = 1..d+1, one pass   (Sec. 3.2.2, Alg. 1)
   4. n_b = number of leading j with argmax p_{b,j} = x_{b,j}           (hard rejection)
+     or with u_{b,j} <= min(1, p_{b,j}(x_{b,j}) / q_{b,j}(x_{b,j}))     (speculative sampling,
+                                                                         Sec. 3.2.2)
      a_b = n_b / d                                                      (acceptance score)
   5. r_b^full = R(T + c_b + x_{b,1..d})  (the CDLH-appx score, Alg. 2)
      r_b^acc  = R(T + c_b + x_{b,1..n_b}) (the S1 score, Alg. 1)
@@ -103,6 +105,20 @@ class Decider:
                 return g
         return best
 
+    def accept(self, log_u: float, log_ratio: float, j: int, kind: str, idx) -> bool:
+        """Speculative-sampling test u <= min(1, p/q), as log u <= log p - log q (u < 1).
+
+        ``other[kind][idx]`` is the other side's accepted count n; its decision for position
+        j is ``j < n``, adopted when this side's margin is within ``tol``."""
+        ok = bool(log_u <= log_ratio)
+        g = self._theirs(kind, idx)
+        if g is not None:
+            theirs = j < int(g)
+            if theirs != ok and abs(log_u - log_ratio) <= self.tol:
+                self.adopted.append((kind, idx, j, ok, theirs))
+                return theirs
+        return ok
+
     def reward_ok(self, r: float, r_t: float, kind: str, idx) -> bool:
         """r >= r_t, compared in float32 (the precision the CUDA path decides in)."""
         ok = bool(np.float32(r) >= np.float32(r_t))
@@ -126,6 +142,35 @@ class RunParams:
     max_new: int                  # l_m of Alg. 1
     composite_reward: bool        # 0.5 coverage + 0.5 sigmoid(w.h) instead of coverage alone
     b: int = 0                    # Step-1 budget of Alg. 1 (literal mode only)
+    acceptance: int = 0           # 0 hard rejection, 1 speculative sampling (Sec. 3.2.2)
+    seed: int = 0                 # seed of the speculative-sampling uniforms
+
+
+HARD, SPECULATIVE = 0, 1
+_MASK64 = (1 << 64) - 1
+
+
+def splitmix64(seed: int, c: int) -> int:
+    """Output number c (from 0) of the SplitMix64 generator seeded with ``seed``.
+
+    SplitMix64 (Steele, Lea, Flood, "Fast splittable pseudorandom number generators", OOPSLA
+    2014): the state advances by the golden-ratio gamma 0x9E3779B97F4A7C15 and each output is
+    the state after that step run through the variant-13 mixer (xor-shift 30, multiply,
+    xor-shift 27, multiply, xor-shift 31)."""
+    z = (seed + (c + 1) * 0x9E3779B97F4A7C15) & _MASK64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _MASK64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _MASK64
+    return z ^ (z >> 31)
+
+
+def uniform24(seed: int, c: int) -> float:
+    """u in [0, 1) with 24 random bits (exact in float32): the top 24 bits of output c."""
+    return (splitmix64(seed, c) >> 40) / float(1 << 24)
+
+
+def draw_index(step: int, B: int, b: int, k: int, beam: int, d: int, j: int) -> int:
+    """Counter of the uniform of prompt b, beam, lookahead position j (0-based) at ``step``."""
+    return ((step * B + b) * k + beam) * d + j
 
 
 def n_min(a_t: float, d: int) -> int:
@@ -217,8 +262,11 @@ class StepRecord:
 
 def cdsl_k_step(target: Transformer, draft: Transformer, states: List[PromptState],
                 run: RunParams, w_head: np.ndarray,
-                decider: Optional[Decider] = None) -> List[StepRecord]:
-    """One CDSL-k step for every prompt that has not reached l_m; updates ``states``."""
+                decider: Optional[Decider] = None, step: int = 0) -> List[StepRecord]:
+    """One CDSL-k step for every prompt that has not reached l_m; updates ``states``.
+
+    ``step`` is the number of steps taken before this one (it indexes the speculative-sampling
+    uniforms)."""
     dec = decider or Decider()
     k, d = run.k, run.d
     nmin = n_min(run.a_t, d)
@@ -272,9 +320,15 @@ def cdsl_k_step(target: Transformer, draft: Transformer, states: List[PromptStat
                                                                    vhid[i, j]))))
             for j in range(d):
                 logp[i, j] = log_softmax(vlog[i, j])[x[b][i, j]]
-            # 4. hard rejection: row j-1 (p_j) must agree with x_j
+            # 4. validation by M_p (Sec. 3.2.2): row j-1 gives p_j for x_j
             for j in range(d):
-                if am[i, j] != x[b][i, j]:
+                if run.acceptance == HARD:        # hard rejection: argmax p_j == x_j
+                    ok = am[i, j] == x[b][i, j]
+                else:                             # speculative sampling: u <= min(1, p/q)
+                    u = uniform24(run.seed, draw_index(step, len(states), b, k, i, d, j))
+                    log_u = np.log(u) if u > 0.0 else -np.inf
+                    ok = dec.accept(log_u, logp[i, j] - logq[b][i, j], j, "spec", (b, i))
+                if not ok:
                     break
                 n[i] += 1
         # 5. rewards
@@ -319,10 +373,10 @@ def cdsl_k_generate(target, draft, prompts, keywords, run: RunParams, w_head,
     """Run CDSL-k steps until every prompt has l_m tokens. Returns (states, records)."""
     states = prefill(target, draft, prompts, keywords)
     records = []
-    for _ in range(max_steps):
+    for step in range(max_steps):
         if all(len(st.T) >= run.max_new for st in states):
             break
-        records.append(cdsl_k_step(target, draft, states, run, w_head))
+        records.append(cdsl_k_step(target, draft, states, run, w_head, step=step))
     return states, records
 
 

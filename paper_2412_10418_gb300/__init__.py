@@ -42,7 +42,8 @@ class RunCfg(ctypes.Structure):
                 ("max_prompt", ctypes.c_int32), ("max_new", ctypes.c_int32),
                 ("n_keywords", ctypes.c_int32), ("a_t", ctypes.c_float), ("r_t", ctypes.c_float),
                 ("reward_head", ctypes.c_int32), ("page_size", ctypes.c_int32),
-                ("max_chunk", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("max_chunk", ctypes.c_int32), ("acceptance", ctypes.c_int32),
+                ("seed", ctypes.c_uint32)]
 
 
 _P = ctypes.c_void_p
@@ -111,10 +112,13 @@ def model_cfg(shape, dtype) -> ModelCfg:
                     shape.norm_eps)
 
 
+ACCEPT_HARD, ACCEPT_SPECULATIVE = 0, 1
+
+
 def run_cfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, reward_head,
-            page_size=0, max_chunk=0) -> RunCfg:
+            page_size=0, max_chunk=0, acceptance=ACCEPT_HARD, seed=0) -> RunCfg:
     return RunCfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, int(reward_head),
-                  page_size, max_chunk, 0)
+                  page_size, max_chunk, int(acceptance), int(seed) & 0xFFFFFFFF)
 
 
 # ------------------------------------------------------------------------------ C names
@@ -222,14 +226,15 @@ class Engine:
 
     def __init__(self, target_shape, draft_shape, dtype, target_weights, draft_weights, *,
                  batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, reward_head=None,
-                 page_size=0, max_chunk=0, stream=None, device="cuda"):
+                 page_size=0, max_chunk=0, acceptance=ACCEPT_HARD, seed=0, stream=None,
+                 device="cuda"):
         import torch
 
         self.torch = torch
         self.tcfg = model_cfg(target_shape, dtype)
         self.dcfg = model_cfg(draft_shape, dtype)
         self.run = run_cfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t,
-                           reward_head is not None, page_size, max_chunk)
+                           reward_head is not None, page_size, max_chunk, acceptance, seed)
         self.B, self.k, self.d, self.V = batch, k, d, target_shape.vocab
         self.max_prompt, self.max_new = max_prompt, max_new
         self.tw, self.dw = list(target_weights), list(draft_weights)

@@ -127,13 +127,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc::tma_load_2d_hint(st, &maps.w[m0], kb * 64, y0, &full_bar[i % S], pol);
     tc::tma_load_2d_hint(st + 8192, &maps.w[m1], kb * 64, y1, &full_bar[i % S], pol);
   };
-  auto load_x = [&](int i, int kb) {
+  auto load_x = [&](int i, int kb) {   // one box of NP rows per plane (the maps' box)
     uint8_t* st = smem + (size_t)(i % S) * stage_bytes;
-    for (int j = 0; j < NP / 16; ++j) {
-      tc::tma_load_2d(st + 16384 + j * 2048, &maps.xh, kb * 64, j * 16, &full_bar[i % S]);
-      tc::tma_load_2d(st + 16384 + NP * 128 + j * 2048, &maps.xl, kb * 64, j * 16,
-                      &full_bar[i % S]);
-    }
+    tc::tma_load_2d(st + 16384, &maps.xh, kb * 64, 0, &full_bar[i % S]);
+    tc::tma_load_2d(st + 16384 + NP * 128, &maps.xl, kb * 64, 0, &full_bar[i % S]);
   };
   if (threadIdx.x == 0) {
     for (int m = 0; m < 3; ++m) tc::tma_prefetch_map(&maps.w[m]);

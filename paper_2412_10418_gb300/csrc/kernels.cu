@@ -291,6 +291,17 @@ __device__ void alloc_pages(const KvStore& kv, int b, int from, int to, int32_t*
 }
 
 // One warp per prompt, one lane per beam: n_b, rewards, b*, state, emission, page allocation.
+// Draw number c of the SplitMix64 generator seeded with `seed` (Steele, Lea, Flood, 2014:
+// state_c = seed + (c + 1) * golden gamma, output = the variant-13 mix of the state), reduced
+// to its top 24 bits as a float in [0, 1) (exact in float32).
+__device__ __forceinline__ float uniform24(uint32_t seed, unsigned long long c) {
+  unsigned long long z = (unsigned long long)seed + (c + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  z ^= z >> 31;
+  return (float)(z >> 40) * (1.0f / 16777216.0f);
+}
+
 __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
   pdl_wait();
   pdl_launch_dependents();
@@ -310,9 +321,19 @@ __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
   int n = 0;
   if (lane < k) {
     const int bi = b * k + lane;
-    for (int j = 0; j < d; ++j) {
-      if (st.v_amax[bi * dp1 + j] != st.x[bi * d + j]) break;
-      ++n;
+    if (st.acceptance == 0) {   // hard rejection: M_p's argmax must equal the drafted token
+      for (int j = 0; j < d; ++j) {
+        if (st.v_amax[bi * dp1 + j] != st.x[bi * d + j]) break;
+        ++n;
+      }
+    } else {                    // speculative sampling: u_j <= min(1, p_j(x_j) / q_j(x_j))
+      const unsigned long long step = (unsigned long long)st.counters[0];
+      const unsigned long long c0 = ((step * st.B + b) * k + lane) * d;
+      for (int j = 0; j < d; ++j) {
+        const float u = uniform24(st.seed, c0 + j);
+        if (!(logf(u) <= st.v_logp[bi * d + j] - st.logq[bi * d + j])) break;
+        ++n;
+      }
     }
     const int root = st.roots[bi];
     uint32_t cf = st.cov[b], ca = st.cov[b];

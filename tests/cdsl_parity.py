@@ -31,12 +31,13 @@ def make_setup(wl: synth.Workload, lens=None, keywords=None, draft_equals_target
     return Setup(wl, t, d, p, lens, kw, synth.reward_head(wl))
 
 
-def run_params(wl: synth.Workload) -> oracle.RunParams:
+def run_params(wl: synth.Workload, acceptance=0, seed=0) -> oracle.RunParams:
     return oracle.RunParams(k=wl.k, d=wl.d, a_t=wl.a_t, r_t=wl.r_t, max_new=wl.max_new,
-                            composite_reward=wl.reward_head)
+                            composite_reward=wl.reward_head, acceptance=acceptance, seed=seed)
 
 
-def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0):
+def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0, acceptance=0,
+                seed=0):
     import torch
     import paper_2412_10418_gb300 as cdsl
 
@@ -53,7 +54,8 @@ def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0):
     eng = cdsl.Engine(wl.target, dshape, wl.dtype, order_t, order_d, batch=wl.batch, k=wl.k,
                       d=wl.d, max_prompt=wl.prompt_len, max_new=wl.max_new,
                       n_keywords=s.keywords.shape[1], a_t=wl.a_t, r_t=wl.r_t, reward_head=head,
-                      page_size=page_size, max_chunk=max_chunk)
+                      page_size=page_size, max_chunk=max_chunk, acceptance=acceptance,
+                      seed=seed)
     eng.prefill(torch.from_numpy(s.prompts), s.lens, torch.from_numpy(s.keywords))
     return eng
 
@@ -125,17 +127,18 @@ def compare_step(g, recs, tol, tol_r, report):
 
 def decider_from(g, tol, tol_r):
     other = {"roots": g["roots"], "x": g["draft_tok"], "argmax": g["argmax"],
-             "beam": g["beam"], "s1": g["state"] == oracle.S1}
+             "beam": g["beam"], "s1": g["state"] == oracle.S1, "spec": g["n_accept"]}
     return oracle.Decider(other=other, tol=tol, tol_r=tol_r)
 
 
 def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_size=16,
-               max_chunk=0):
+               max_chunk=0, acceptance=0, seed=0):
     """Step the GPU and the oracle together; every step is compared element by element."""
-    eng = eng or make_engine(s, page_size=page_size, max_chunk=max_chunk)
+    eng = eng or make_engine(s, page_size=page_size, max_chunk=max_chunk, acceptance=acceptance,
+                             seed=seed)
     tgt, drf = oracle_models(s)
     states = oracle_prefill(s, tgt, drf)
-    run = run_params(s.wl)
+    run = run_params(s.wl, acceptance, seed)
     report: Dict[str, float] = {}
     adopted = []
     n_steps = 0
@@ -144,8 +147,10 @@ def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_si
             break
         g = gpu_step_outputs(eng)
         dec = decider_from(g, tol, tol_r)
-        recs = oracle.cdsl_k_step(tgt, drf, states, run, s.w_head, dec)
+        recs = oracle.cdsl_k_step(tgt, drf, states, run, s.w_head, dec, step=n_steps)
         compare_step(g, recs, tol, tol_r, report)
+        report["accepted"] = report.get("accepted", 0) + int(
+            sum(g["n_accept"][b].sum() for b, r in enumerate(recs) if r.active))
         adopted += dec.adopted
         n_steps += 1
     assert eng.status() == 0

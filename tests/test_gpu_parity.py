@@ -142,3 +142,55 @@ def test_nonfinite_logits_are_flagged():
     eng = make_engine(s, torch_weights=(tw, dw))
     eng.lookahead(); eng.verify(); eng.select()
     assert eng.status() == 5
+
+
+@pytest.mark.parametrize("seed", [1, 7])
+def test_tiny_speculative_sampling(seed):
+    """Speculative-sampling validation (Sec. 3.2.2): n_b from u <= min(1, p/q) with the
+    SplitMix64 uniforms both sides draw from the same counters."""
+    wl = synth.scaled(synth.TINY, batch=2, max_new=24)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=24, tol=TOL32, tol_r=TOL32,
+                                              acceptance=oracle.SPECULATIVE, seed=seed)
+    tokens_match(eng, states)
+    assert rep["accepted"] > 0      # some drafted tokens passed u <= p/q
+    print("speculative sampling", seed, "max |diff|:", rep, "adopted:", len(adopted))
+
+
+def test_tiny_speculative_sampling_draft_equals_target():
+    """M_q = M_p: p/q = 1 at every drafted token, so every lookahead is accepted in full."""
+    wl = synth.scaled(synth.TINY, draft=synth.TINY.target, max_new=20)
+    s = make_setup(wl, draft_equals_target=True)
+    eng, states, rep, adopted, n = run_parity(s, steps=20, tol=TOL32, tol_r=TOL32,
+                                              acceptance=oracle.SPECULATIVE, seed=3)
+    tokens_match(eng, states)
+    g = gpu_step_outputs(eng)
+    if g["n_emitted"].sum() > 0:
+        assert np.all(g["n_accept"][g["n_emitted"] > 0] == wl.d)
+
+
+def test_small_bf16_speculative_sampling():
+    wl = synth.scaled(synth.SMALL, batch=2, max_new=16)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=4, tol=TOL16, tol_r=TOL16,
+                                              acceptance=oracle.SPECULATIVE, seed=11)
+    tokens_match(eng, states)
+    assert rep["accepted"] > 0
+    print("bf16 speculative sampling max |diff|:", rep, "adopted:", len(adopted))
+
+
+def test_tiny_cdlh_on_the_same_kernels():
+    """Alg. 2 CDLH on the GPU path: M_p drafts its own lookaheads and no reward reaches r_t,
+    so every step emits one token: the CDLH token of the oracle's Alg. 2 (Sec. 3.1), step by
+    step and over the whole generation."""
+    wl = synth.scaled(synth.TINY, draft=synth.TINY.target, r_t=2.0, max_new=10)
+    s = make_setup(wl, draft_equals_target=True)
+    eng, states, rep, adopted, n = run_parity(s, steps=10, tol=TOL32, tol_r=TOL32)
+    assert n == wl.max_new                # one token per step
+    tokens_match(eng, states)
+    tgt = oracle.Transformer(wl.target, s.t_host)
+    run = run_params(wl)
+    for b in range(wl.batch):
+        ref = oracle.cdlh_generate(tgt, tgt, tgt, s.prompts[b].tolist(), s.keywords[b].tolist(),
+                                   run, s.w_head)
+        assert states[b].T == ref.T

@@ -276,3 +276,81 @@ def test_tiny_workload_runs():
                                           synth.reward_head(wl))
     assert len(states[0].T) == wl.max_new
     assert all(len(r[0].emitted) >= 1 for r in recs)
+
+
+# ---------------------------------------------------------------- speculative sampling (f1)
+
+def test_splitmix64_published_outputs():
+    """The generator behind the speculative-sampling uniforms matches SplitMix64's published
+    check values (seed 1234567)."""
+    vals = [int(x) for x in open(os.path.join(GOLDEN, "splitmix64_seed1234567.txt"))
+            if x.strip() and not x.startswith("#")]
+    seed, want = vals[0], vals[1:]
+    assert [oracle.splitmix64(seed, c) for c in range(len(want))] == want
+
+
+def test_uniform24_is_uniform_and_float32_exact():
+    """u = top 24 bits / 2^24: in [0, 1), exactly representable in float32, and uniform
+    (mean and a 16-bin chi-square over 2^16 draws)."""
+    n = 1 << 16
+    u = np.array([oracle.uniform24(12345, c) for c in range(n)])
+    assert np.all((u >= 0.0) & (u < 1.0))
+    assert np.array_equal(u.astype(np.float32).astype(np.float64), u)
+    assert abs(u.mean() - 0.5) < 4 * np.sqrt(1 / 12 / n)
+    counts = np.bincount((u * 16).astype(int), minlength=16)
+    chi2 = float(np.sum((counts - n / 16) ** 2 / (n / 16)))
+    assert chi2 < 45.0          # 15 degrees of freedom: p ~ 1e-4
+
+
+@pytest.mark.parametrize("rho", [0.1, 0.5, 0.9])
+def test_speculative_test_accepts_with_probability_p_over_q(rho):
+    """Sec. 3.2.2: a token is rejected when r > min(1, p/q), r ~ U[0, 1]; so it is accepted
+    with probability p/q (< 1). The decision on the draws of one generator matches that
+    frequency (a flipped inequality would give 1 - p/q)."""
+    n = 40000
+    dec = Decider()
+    acc = sum(dec.accept(np.log(u) if u > 0 else -np.inf, np.log(rho), 0, "spec", None)
+              for u in (oracle.uniform24(99, c) for c in range(n)))
+    assert abs(acc / n - rho) < 4 * np.sqrt(rho * (1 - rho) / n)
+
+
+def test_speculative_identical_models_accept_everything():
+    """M_q = M_p under speculative sampling: p/q = 1 at every drafted token, every lookahead
+    is accepted in full whatever the uniforms."""
+    shp = shape(vocab=40)
+    tgt = model(shp, 1)
+    run = run_params(k=3, d=4, r_t=10.0, acceptance=oracle.SPECULATIVE, seed=5)
+    st = prefill(tgt, tgt, np.array([[1, 2, 3, 4, 5], [9, 8, 7, 6, 5]]), np.array([[1, 2], [3, 4]]))
+    w = np.random.default_rng(2).standard_normal(shp.d_model)
+    for step in range(3):
+        for rec in cdsl_k_step(tgt, tgt, st, run, w, step=step):
+            assert np.all(rec.n == run.d)
+
+
+def test_speculative_draws_follow_the_counter():
+    """The uniform of (step, prompt, beam, position) is draw number
+    ((step * B + b) * k + beam) * d + j: distinct for every decision of a run."""
+    B, k, d = 3, 4, 5
+    idx = {oracle.draw_index(s, B, b, k, i, d, j) for s in range(4) for b in range(B)
+           for i in range(k) for j in range(d)}
+    assert idx == set(range(4 * B * k * d))
+
+
+def test_speculative_vs_hard_on_different_models():
+    """Different models: the speculative count never exceeds the draws' verdicts, i.e. every
+    accepted position j has u_j <= p_j/q_j, and the first rejected one (if any) has
+    u_j > p_j/q_j."""
+    shp = shape(vocab=24)
+    tgt, drf = model(shp, 1), model(shp, 2)
+    run = run_params(k=3, d=4, acceptance=oracle.SPECULATIVE, seed=17)
+    st = prefill(tgt, drf, np.array([[1, 2, 3, 4, 5, 6]]), np.array([[1, 2]]))
+    w = np.random.default_rng(2).standard_normal(shp.d_model)
+    for step in range(4):
+        for rec in cdsl_k_step(tgt, drf, st, run, w, step=step):
+            if not rec.active:
+                continue
+            for i in range(run.k):
+                for j in range(min(rec.n[i] + 1, run.d)):
+                    u = oracle.uniform24(run.seed, oracle.draw_index(step, 1, 0, run.k, i, run.d, j))
+                    ratio = np.exp(rec.logp[i, j] - rec.logq[i, j])
+                    assert (u <= ratio) == (j < rec.n[i])
