@@ -100,6 +100,18 @@ __device__ __forceinline__ float4 ld_cluster_f32x4(uint32_t addr) {
   return v;
 }
 
+// ------------------------------------------------------------------------------ global
+// Atomic add with acquire-release semantics at GPU scope; returns the old value. After a
+// block barrier, one thread's release is cumulative: it publishes the whole block's prior
+// writes; its acquire, followed by a block barrier, makes the other blocks' published
+// writes visible to the whole block.
+__device__ __forceinline__ int atom_add_acq_rel_gpu(int* p, int v) {
+  int old;
+  asm volatile("atom.add.acq_rel.gpu.global.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v)
+               : "memory");
+  return old;
+}
+
 // ------------------------------------------------------------------------------ TMA
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
