@@ -14,11 +14,10 @@
 // query vectors, and writes the normalized output in the GEMM-input format. No global scratch,
 // no atomics.
 //
-// Per chunk: S = Q K^T and o += P V run on the tensor cores in 3xTF32 (mma.sync m16n8k8, each
-// fp32 operand split into a tf32 high part and a tf32 remainder: fp32-level accuracy), their
-// 16x8 tiles spread evenly over the 8 warps; the online softmax between them runs on the CUDA
-// cores, a warp owning QPW (2 or 4) query vectors and its lanes keys lane and lane + 32. A
-// query block is 8 * QPW query vectors.
+// Score loop: a warp owns QPW (2, 4 or 5) query vectors (broadcast reads), its lanes own keys lane
+// and lane + 32 (rows of 132 floats: conflict-free 128-bit reads). Output loop: lanes own 4
+// (or 2) consecutive dims of the warp's query vectors, reading P by broadcast and V
+// row-contiguously. All 8 warps have query vectors: a query block is 8 * QPW of them.
 #include <algorithm>
 
 #include <cooperative_groups.h>
@@ -31,7 +30,7 @@ namespace {
 namespace cg = cooperative_groups;
 
 constexpr int ACH = 64;              // key slots per chunk
-constexpr int AQB = 32;              // query vectors per cluster (at most)
+constexpr int AQB = 40;              // query vectors per cluster (at most)
 constexpr int MAXP = 64;             // chunks (prefix + tail) of a pass
 constexpr int ACL = 16;              // blocks per cluster (at most)
 constexpr int MAXCB = MAXP / 8;      // chunks per block (at most; clusters have >= 8 blocks
@@ -43,60 +42,11 @@ int g_max_cluster = 8;               // 16 where non-portable clusters of this k
 
 template <int HD>
 struct AttnSmem {
-  static constexpr int QP = HD + 4;        // row pitch of Q and K (conflict-free fragments)
-  static constexpr int VP = HD + 8;        // row pitch of V
-  static constexpr int SP = ACH + 4;       // row pitch of the scores / probabilities
-  static constexpr size_t floats = (size_t)AQB * QP + (size_t)ACH * QP + (size_t)ACH * VP + (size_t)AQB * SP;
+  static constexpr int QP = HD + 4;        // padded row pitch of Q and K
+  static constexpr int PP = AQB + 4;       // row pitch of P (4-way store conflicts at most)
+  static constexpr size_t floats = (size_t)AQB * QP + (size_t)ACH * QP + (size_t)ACH * HD + (size_t)ACH * PP;
   static constexpr size_t bytes = floats * sizeof(float);
 };
-
-// ---- 3xTF32 tensor-core products (mma.sync m16n8k8): x = hi + lo with hi = tf32(x),
-//      lo = tf32(x - hi); a.b ~ a_hi.b_hi + a_hi.b_lo + a_lo.b_hi (the a_lo.b_lo term and the
-//      rounding of the lo parts are below 2^-21 relative: fp32-level accuracy)
-__device__ __forceinline__ void split_tf32(float x, uint32_t& hi, uint32_t& lo) {
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(hi) : "f"(x));
-  const float rest = x - __uint_as_float(hi);
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(lo) : "f"(rest));
-}
-__device__ __forceinline__ void mma_tf32(float (&d)[4], const uint32_t (&a)[4], const uint32_t (&b)[2]) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-      "{%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
-}
-// Fragments of one 16x8x8 step, split into tf32 high and low parts: A from a row-major [m][k]
-// tile (element (m, k) at A[m * lda + k]); B from a [n][k] tile (B[n * ldb + k]) or, with kn,
-// a [k][n] tile (B[k * ldb + n]).
-struct FragA { uint32_t h[4], l[4]; };
-struct FragB { uint32_t h[2], l[2]; };
-__device__ __forceinline__ FragA load_a(const float* A, int lda, int lane) {
-  const int g = lane >> 2, t = lane & 3;
-  FragA f;
-  split_tf32(A[g * lda + t], f.h[0], f.l[0]);
-  split_tf32(A[(g + 8) * lda + t], f.h[1], f.l[1]);
-  split_tf32(A[g * lda + t + 4], f.h[2], f.l[2]);
-  split_tf32(A[(g + 8) * lda + t + 4], f.h[3], f.l[3]);
-  return f;
-}
-template <bool kn>
-__device__ __forceinline__ FragB load_b(const float* B, int ldb, int lane) {
-  const int g = lane >> 2, t = lane & 3;
-  FragB f;
-  if (kn) {
-    split_tf32(B[t * ldb + g], f.h[0], f.l[0]);
-    split_tf32(B[(t + 4) * ldb + g], f.h[1], f.l[1]);
-  } else {
-    split_tf32(B[g * ldb + t], f.h[0], f.l[0]);
-    split_tf32(B[g * ldb + t + 4], f.h[1], f.l[1]);
-  }
-  return f;
-}
-__device__ __forceinline__ void mma3(float (&d)[4], const FragA& a, const FragB& b) {
-  mma_tf32(d, a.l, b.h);   // small terms first
-  mma_tf32(d, a.h, b.l);
-  mma_tf32(d, a.h, b.h);
-}
 
 template <typename T, int HD, int QPW>
 __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
@@ -105,14 +55,14 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   extern __shared__ float4 sm4[];
   float* qS = reinterpret_cast<float*>(sm4);   // [QB][QP]  pre-scaled queries
   float* kS = qS + AQB * L::QP;                 // [ACH][QP]; after the chunks: partial o [QB][HD]
-  float* vS = kS + ACH * L::QP;                 // [ACH][VP]
-  float* pS = vS + ACH * L::VP;                 // [QB][SP] scores, then probabilities
+  float* vS = kS + ACH * L::QP;                 // [ACH][HD]
+  float* pS = vS + ACH * HD;                    // [ACH][PP] probabilities
   __shared__ int s_row[QB], s_gg[QB], s_np[QB], s_tb[QB], s_nt[QB];
-  __shared__ int s_toff[32], s_tlen[32];        // per query vector: its tail's slot range
+  __shared__ int s_toff[32], s_tlen[32], s_ttb[32];   // per row of the block: its tail's
+                                                      // slot range (first row of a tail only)
   __shared__ int s_wcnt[AWARPS];
   __shared__ int s_nrows, s_maxnp;
-  __shared__ float s_pm[QB], s_pl[QB];          // running (m, l) per query vector
-  __shared__ float s_alpha[QB];                 // this chunk's rescale of o per query vector
+  __shared__ float s_pm[QB], s_pl[QB];          // the block's partial (m, l) per query vector
   __shared__ const float* s_kp[MAXCB * ACH];    // K row of every key slot of the block's chunks
   __shared__ int s_ktb[MAXCB * ACH];            // tail slots: tail base of the beam,
   __shared__ uint8_t s_kj[MAXCB * ACH];         //   index in it
@@ -173,13 +123,17 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   }
   const int nq = max(0, min(QB, s_nrows * G - qb * QB));
   if (warp == 0) {
-    // longest prefix, and the distinct tails (lane = query vector) in order of first
-    // appearance, each as long as its longest row: slot offsets in their concatenation
-    int np = (lane < nq) ? s_np[lane] : 0;
+    // longest prefix, and the distinct tails (lane = row of the block: at most 32, see
+    // attn_qblock_for) in order of first appearance, each as long as its longest row: slot
+    // offsets in their concatenation
+    const int first_local = (qb * QB) / G;
+    const int qi_l = max(0, (first_local + lane) * G - qb * QB);   // the row's first vector
+    const bool row_ok = nq > 0 && qi_l < nq && lane <= (qb * QB + nq - 1) / G - first_local;
+    int np = row_ok ? s_np[qi_l] : 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) np = max(np, __shfl_xor_sync(0xffffffffu, np, o));
-    const int tb = (lane < nq) ? s_tb[lane] : -1;
-    const int nt = (lane < nq) ? s_nt[lane] : 0;
+    const int tb = row_ok ? s_tb[qi_l] : -1;
+    const int nt = row_ok ? s_nt[qi_l] : 0;
     int len = 0;
     bool first = nt > 0;
     for (int j = 0; j < 32; ++j) {
@@ -199,6 +153,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     const int total = __shfl_sync(0xffffffffu, off, 31);
     s_toff[lane] = off - len;
     s_tlen[lane] = len;
+    s_ttb[lane] = tb;
     if (lane == 0) {
       s_maxnp = np;
       if (cx == 0 && total > a.n_tchunks * ACH) set_status(a.status, CDSL_ERANGE);
@@ -217,8 +172,8 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
           s_kp[i * ACH + threadIdx.x] = a.kv.pool + kv_prefix_offset(a.kv, a.layer, page, 0, g,
                                                                      t & ((1 << a.kv.page_shift) - 1));
       }
-    } else if (warp == 0 && lane < nq) {   // tail slots [lo, lo + 64) of the concatenation
-      const int lo = (c - n_p) * ACH, off = s_toff[lane], len = s_tlen[lane], tb = s_tb[lane];
+    } else if (warp == 0) {   // tail slots [lo, lo + 64) of the concatenation
+      const int lo = (c - n_p) * ACH, off = s_toff[lane], len = s_tlen[lane], tb = s_ttb[lane];
       for (int e = max(0, lo - off); e < len && off + e < lo + ACH; ++e) {
         const int sl = i * ACH + off + e - lo;
         s_kp[sl] = a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, tb + e, g);
@@ -232,21 +187,15 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   pdl_launch_dependents();
 
   constexpr int DPL = HD / 32;
-  const int q0 = warp * QPW;      // softmax rows of this warp
-  // tensor-core tiles: scores QB x 64 and outputs QB x HD in 16x8 tiles, spread evenly over
-  // the 8 warps (a warp's tiles share their 16 query rows)
-  constexpr int MT = QB / 16;
-  constexpr int ST = MT * (ACH / 8) / AWARPS;   // score tiles per warp
-  constexpr int OT = MT * (HD / 8) / AWARPS;    // output tiles per warp
-  const int s_m = (warp * ST) / (ACH / 8), s_n0 = (warp * ST) % (ACH / 8);
-  const int o_m = (warp * OT) / (HD / 8), o_n0 = (warp * OT) % (HD / 8);
-  const int fg = lane >> 2, ft = lane & 3;      // fragment row group, column pair
-  float oacc[OT][4];                            // rows o_m*16 + fg (+8), cols n*8 + 2*ft (+1)
+  const int q0 = warp * QPW;
+  const bool active = q0 < nq;   // warps without query vectors only help to stage
+  float o[QPW][DPL], m_run[QPW], l_run[QPW];
 #pragma unroll
-  for (int i = 0; i < OT; ++i) oacc[i][0] = oacc[i][1] = oacc[i][2] = oacc[i][3] = 0.f;
-  if (threadIdx.x < QB) {
-    s_pm[threadIdx.x] = -INFINITY;
-    s_pl[threadIdx.x] = 0.f;
+  for (int i = 0; i < QPW; ++i) {
+    m_run[i] = -INFINITY;
+    l_run[i] = 0.f;
+#pragma unroll
+    for (int c = 0; c < DPL; ++c) o[i][c] = 0.f;
   }
   bool q_staged = false;
   for (int i = 0; i < nb_chunks && nq > 0; ++i) {
@@ -256,7 +205,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     if (!tail && t0 >= maxnp) continue;   // beyond every query vector's prefix
     // ---- stage K and V of the chunk's 64 slots (and Q the first time), loads in flight
     //      together
-    constexpr int QPER = QB * (HD / 4) / ATHREADS;
+    constexpr int QPER = (QB * (HD / 4) + ATHREADS - 1) / ATHREADS;   // (last pass partial)
     constexpr int PER = ACH * (HD / 4) / ATHREADS;   // float4 per thread per matrix
     const size_t v_delta = tail ? (size_t)a.kv.n_tail_slots * a.kv.kvh * HD
                                 : ((size_t)a.kv.kvh << a.kv.page_shift) * HD;
@@ -267,7 +216,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         const int idx = threadIdx.x + u * ATHREADS;
         const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
         qr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (qi < nq)
+        if (qi < nq && qi < QB)
           qr[u] = *reinterpret_cast<const float4*>(a.q + (size_t)s_row[qi] * H * HD +
                                                    (size_t)(g * G + s_gg[qi]) * HD + 4 * e4);
       }
@@ -291,7 +240,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
         float4 v = qr[u];
         v.x *= a.scale; v.y *= a.scale; v.z *= a.scale; v.w *= a.scale;
-        *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
+        if (qi < QB) *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
       }
       q_staged = true;
     }
@@ -300,38 +249,31 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
       const int idx = threadIdx.x + u * ATHREADS;
       const int j = idx / (HD / 4), e4 = idx % (HD / 4);
       *reinterpret_cast<float4*>(kS + j * L::QP + 4 * e4) = kr[u];
-      *reinterpret_cast<float4*>(vS + j * L::VP + 4 * e4) = vr[u];
+      *reinterpret_cast<float4*>(vS + j * HD + 4 * e4) = vr[u];
     }
     __syncthreads();
+    if (!active) continue;
 
-    // ---- scores S = Q K^T on the tensor cores (3xTF32): Q rows s_m*16.., keys n*8..
-    {
-      float sacc[ST][4];
+    // ---- scores: warp -> QPW query vectors, lane -> keys lane, lane + 32
+    float s[QPW][2];
 #pragma unroll
-      for (int i = 0; i < ST; ++i) sacc[i][0] = sacc[i][1] = sacc[i][2] = sacc[i][3] = 0.f;
+    for (int q = 0; q < QPW; ++q) s[q][0] = s[q][1] = 0.f;
 #pragma unroll 4
-      for (int k0 = 0; k0 < HD; k0 += 8) {
-        const FragA fa = load_a(qS + (s_m * 16) * L::QP + k0, L::QP, lane);
+    for (int e = 0; e < HD; e += 4) {
+      const float4 k0 = *reinterpret_cast<const float4*>(kS + lane * L::QP + e);
+      const float4 k1 = *reinterpret_cast<const float4*>(kS + (lane + 32) * L::QP + e);
 #pragma unroll
-        for (int i = 0; i < ST; ++i)
-          mma3(sacc[i], fa, load_b<false>(kS + ((s_n0 + i) * 8) * L::QP + k0, L::QP, lane));
-      }
-#pragma unroll
-      for (int i = 0; i < ST; ++i) {
-        float* dst = pS + (s_m * 16 + fg) * L::SP + (s_n0 + i) * 8 + 2 * ft;
-        dst[0] = sacc[i][0];
-        dst[1] = sacc[i][1];
-        dst[8 * L::SP] = sacc[i][2];
-        dst[8 * L::SP + 1] = sacc[i][3];
+      for (int q = 0; q < QPW; ++q) {
+        const float4 qv = *reinterpret_cast<const float4*>(qS + (q0 + q) * L::QP + e);
+        s[q][0] += qv.x * k0.x + qv.y * k0.y + qv.z * k0.z + qv.w * k0.w;
+        s[q][1] += qv.x * k1.x + qv.y * k1.y + qv.z * k1.z + qv.w * k1.w;
       }
     }
-    __syncthreads();
-
-    // ---- online softmax over the chunk: warp -> QPW query vectors, lane -> keys lane, lane+32
+    // ---- online softmax: running max, rescale of l and o, probabilities of this chunk
+    float p0[QPW], p1[QPW];
 #pragma unroll
     for (int q = 0; q < QPW; ++q) {
       const int qi = q0 + q;
-      float* srow = pS + qi * L::SP;
       bool ok0, ok1;
       if (qi >= nq) {
         ok0 = ok1 = false;
@@ -344,55 +286,81 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         ok0 = s_kp[k0] && s_ktb[k0] == tb && s_kj[k0] < nt;
         ok1 = s_kp[k1] && s_ktb[k1] == tb && s_kj[k1] < nt;
       }
-      const float a0 = ok0 ? srow[lane] : -INFINITY, a1 = ok1 ? srow[lane + 32] : -INFINITY;
-      const float m_old = s_pm[qi];
-      const float m_new = fmaxf(m_old, warp_max(fmaxf(a0, a1)));
-      float alpha = 1.f, p0 = 0.f, p1 = 0.f;
+      const float a0 = ok0 ? s[q][0] : -INFINITY, a1 = ok1 ? s[q][1] : -INFINITY;
+      const float m_new = fmaxf(m_run[q], warp_max(fmaxf(a0, a1)));
+      float alpha = 1.f;
+      p0[q] = p1[q] = 0.f;
       if (m_new > -INFINITY) {
-        alpha = (m_old > -INFINITY) ? expf(m_old - m_new) : 0.f;
-        p0 = ok0 ? expf(a0 - m_new) : 0.f;
-        p1 = ok1 ? expf(a1 - m_new) : 0.f;
+        alpha = (m_run[q] > -INFINITY) ? expf(m_run[q] - m_new) : 0.f;
+        p0[q] = ok0 ? expf(a0 - m_new) : 0.f;
+        p1[q] = ok1 ? expf(a1 - m_new) : 0.f;
       }
-      const float psum = warp_sum(p0 + p1);
-      srow[lane] = p0;
-      srow[lane + 32] = p1;
-      if (lane == 0) {
-        s_pl[qi] = alpha * s_pl[qi] + psum;
-        s_pm[qi] = m_new;
-        s_alpha[qi] = alpha;
+      l_run[q] = alpha * l_run[q] + warp_sum(p0[q] + p1[q]);
+      m_run[q] = m_new;
+#pragma unroll
+      for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] *= alpha;
+    }
+    if constexpr (QPW == 4) {
+      *reinterpret_cast<float4*>(pS + lane * L::PP + q0) = make_float4(p0[0], p0[1], p0[2], p0[3]);
+      *reinterpret_cast<float4*>(pS + (lane + 32) * L::PP + q0) =
+          make_float4(p1[0], p1[1], p1[2], p1[3]);
+    } else if constexpr (QPW == 2) {
+      *reinterpret_cast<float2*>(pS + lane * L::PP + q0) = make_float2(p0[0], p0[1]);
+      *reinterpret_cast<float2*>(pS + (lane + 32) * L::PP + q0) = make_float2(p1[0], p1[1]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < QPW; ++q) {
+        pS[lane * L::PP + q0 + q] = p0[q];
+        pS[(lane + 32) * L::PP + q0 + q] = p1[q];
       }
     }
-    __syncthreads();
+    __syncwarp();
 
-    // ---- o = alpha o + P V on the tensor cores (3xTF32): rows o_m*16.., dims n*8..
-    {
-      const float al0 = s_alpha[o_m * 16 + fg], al1 = s_alpha[o_m * 16 + fg + 8];
+    // ---- o += P V: lane -> dims [DPL*lane, DPL*lane + DPL)
+#pragma unroll 4
+    for (int t = 0; t < ACH; ++t) {
+      float pp[QPW];
+      if constexpr (QPW == 4) {
+        const float4 p4 = *reinterpret_cast<const float4*>(pS + t * L::PP + q0);
+        pp[0] = p4.x; pp[1] = p4.y; pp[2] = p4.z; pp[3] = p4.w;
+      } else if constexpr (QPW == 2) {
+        const float2 p2 = *reinterpret_cast<const float2*>(pS + t * L::PP + q0);
+        pp[0] = p2.x; pp[1] = p2.y;
+      } else {
 #pragma unroll
-      for (int n = 0; n < OT; ++n) {
-        oacc[n][0] *= al0; oacc[n][1] *= al0;
-        oacc[n][2] *= al1; oacc[n][3] *= al1;
+        for (int q = 0; q < QPW; ++q) pp[q] = pS[t * L::PP + q0 + q];
       }
-#pragma unroll 2
-      for (int k0 = 0; k0 < ACH; k0 += 8) {
-        const FragA fa = load_a(pS + (o_m * 16) * L::SP + k0, L::SP, lane);
+      float v[DPL];
+      if constexpr (DPL == 4) {
+        const float4 v4 = *reinterpret_cast<const float4*>(vS + t * HD + 4 * lane);
+        v[0] = v4.x; v[1] = v4.y; v[2] = v4.z; v[3] = v4.w;
+      } else {
+        const float2 v2 = *reinterpret_cast<const float2*>(vS + t * HD + 2 * lane);
+        v[0] = v2.x; v[1] = v2.y;
+      }
 #pragma unroll
-        for (int n = 0; n < OT; ++n)
-          mma3(oacc[n], fa, load_b<true>(vS + k0 * L::VP + (o_n0 + n) * 8, L::VP, lane));
-      }
+      for (int q = 0; q < QPW; ++q)
+#pragma unroll
+        for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] = fmaf(pp[q], v[c2], o[q][c2]);
     }
+    __syncwarp();   // pS columns of this warp are rewritten by its next chunk
   }
 
-  // ---- the block's partial o per query vector into shared memory (over kS); (m, l) are in
-  //      s_pm / s_pl
+  // ---- the block's partial (m, l, o) per query vector into shared memory (o over kS)
   __syncthreads();
   float* s_po = kS;
+  if (active) {
 #pragma unroll
-  for (int n = 0; n < OT; ++n) {
-    float* dst = s_po + (o_m * 16 + fg) * HD + (o_n0 + n) * 8 + 2 * ft;
-    dst[0] = oacc[n][0];
-    dst[1] = oacc[n][1];
-    dst[8 * HD] = oacc[n][2];
-    dst[8 * HD + 1] = oacc[n][3];
+    for (int q = 0; q < QPW; ++q) {
+      const int qi = q0 + q;
+      if (qi >= nq) continue;
+#pragma unroll
+      for (int c2 = 0; c2 < DPL; ++c2) s_po[qi * HD + DPL * lane + c2] = o[q][c2];
+      if (lane == 0) {
+        s_pm[qi] = m_run[q];
+        s_pl[qi] = l_run[q];
+      }
+    }
   }
   cluster.sync();   // every block's partials are visible to the cluster
 
@@ -481,9 +449,16 @@ int configure_t() {
 
 int attn_chunk() { return ACH; }
 int attn_max_chunks() { return MAXP; }
-int attn_qblock() { return AQB; }
+int attn_qblock() { return AWARPS * 4; }
 int attn_qblock_for(int rows_per_prompt, int G) {
-  return rows_per_prompt * G <= AWARPS * 2 ? AWARPS * 2 : AQB;
+  // 8 warps x 2, 4 or 5 query vectors: the fewest query blocks (each of them loads the K/V
+  // chunks once), the smallest block that still takes them. Blocks of 40 need G >= 2 (at most
+  // 32 rows per block: the tail layout runs one lane per row).
+  const int nq = rows_per_prompt * G;
+  if (nq <= AWARPS * 2) return AWARPS * 2;
+  if (nq <= AWARPS * 4 || G < 2) return AWARPS * 4;
+  const int n_qb = (nq + AQB - 1) / AQB;
+  return (nq + n_qb - 1) / n_qb <= AWARPS * 4 ? AWARPS * 4 : AQB;
 }
 
 int attn_tail_chunks(int rows_per_prompt, int G, int rows_per_tail, int max_tail) {
@@ -498,9 +473,11 @@ int attn_tail_chunks(int rows_per_prompt, int G, int rows_per_tail, int max_tail
 int configure_attention() {
   int worst = 0;
   for (int r : {configure_t<float, 64, 2>(), configure_t<float, 64, 4>(),
-                configure_t<float, 128, 2>(), configure_t<float, 128, 4>(),
+                configure_t<float, 64, 5>(), configure_t<float, 128, 2>(),
+                configure_t<float, 128, 4>(), configure_t<float, 128, 5>(),
                 configure_t<__nv_bfloat16, 64, 2>(), configure_t<__nv_bfloat16, 64, 4>(),
-                configure_t<__nv_bfloat16, 128, 2>(), configure_t<__nv_bfloat16, 128, 4>()}) {
+                configure_t<__nv_bfloat16, 64, 5>(), configure_t<__nv_bfloat16, 128, 2>(),
+                configure_t<__nv_bfloat16, 128, 4>(), configure_t<__nv_bfloat16, 128, 5>()}) {
     if (r < 0) return -1;
     worst = std::max(worst, r);
   }
@@ -508,14 +485,20 @@ int configure_attention() {
   return 0;
 }
 
+template <typename T, int HD>
+void launch_hd(const AttnArgs& a, int n_z, cudaStream_t s) {
+  if (a.qblock <= AWARPS * 2) launch_t<T, HD, 2>(a, n_z, s);
+  else if (a.qblock <= AWARPS * 4) launch_t<T, HD, 4>(a, n_z, s);
+  else launch_t<T, HD, 5>(a, n_z, s);
+}
+
 void launch_attn(int dtype, const AttnArgs& a, int n_z, cudaStream_t s) {
-  const bool q2 = a.qblock <= AWARPS * 2;
   if (dtype == CDSL_DTYPE_BF16) {
-    if (a.kv.hd == 128) q2 ? launch_t<__nv_bfloat16, 128, 2>(a, n_z, s) : launch_t<__nv_bfloat16, 128, 4>(a, n_z, s);
-    else q2 ? launch_t<__nv_bfloat16, 64, 2>(a, n_z, s) : launch_t<__nv_bfloat16, 64, 4>(a, n_z, s);
+    if (a.kv.hd == 128) launch_hd<__nv_bfloat16, 128>(a, n_z, s);
+    else launch_hd<__nv_bfloat16, 64>(a, n_z, s);
   } else {
-    if (a.kv.hd == 128) q2 ? launch_t<float, 128, 2>(a, n_z, s) : launch_t<float, 128, 4>(a, n_z, s);
-    else q2 ? launch_t<float, 64, 2>(a, n_z, s) : launch_t<float, 64, 4>(a, n_z, s);
+    if (a.kv.hd == 128) launch_hd<float, 128>(a, n_z, s);
+    else launch_hd<float, 64>(a, n_z, s);
   }
 }
 

@@ -194,3 +194,15 @@ def test_tiny_cdlh_on_the_same_kernels():
         ref = oracle.cdlh_generate(tgt, tgt, tgt, s.prompts[b].tolist(), s.keywords[b].tolist(),
                                    run, s.w_head)
         assert states[b].T == ref.T
+
+
+def test_tiny_gqa_wide_query_blocks():
+    """Grouped-query attention (2 query heads per KV head): the 4 x 5 verify rows make 40 query
+    vectors per KV head, taken by one block of 40 (5 per warp); the draft rows by blocks of 16
+    and 32. Ragged batch."""
+    tgt = synth.ModelShape(n_layers=2, d_model=256, n_heads=4, n_kv_heads=2, d_ffn=688, vocab=512)
+    drf = synth.ModelShape(n_layers=1, d_model=128, n_heads=2, n_kv_heads=1, d_ffn=344, vocab=512)
+    wl = synth.scaled(synth.TINY, target=tgt, draft=drf, batch=2, prompt_len=40, max_new=16)
+    s = make_setup(wl, lens=[40, 23])
+    eng, states, rep, adopted, n = run_parity(s, steps=16, tol=TOL32, tol_r=TOL32)
+    tokens_match(eng, states)
