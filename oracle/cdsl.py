@@ -230,8 +230,8 @@ def prefill(target: Transformer, draft: Transformer, prompts: np.ndarray,
     B = prompts.shape[0]
     tcs = [target.new_cache() for _ in range(B)]
     dcs = [draft.new_cache() for _ in range(B)]
-    tl, th = target.forward([(tcs[b], prompts[b].tolist()) for b in range(B)])
-    dl, _ = draft.forward([(dcs[b], prompts[b].tolist()) for b in range(B)])
+    tl, th = target.forward([(tcs[b], prompts[b].tolist()) for b in range(B)], last_only=True)
+    dl, _ = draft.forward([(dcs[b], prompts[b].tolist()) for b in range(B)], last_only=True)
     return [PromptState(prompt=prompts[b].tolist(), T=[], keywords=keywords[b], tcache=tcs[b],
                         dcache=dcs[b], p_root=tl[b][-1], h_root=th[b][-1],
                         q_root=dl[b][-1] if keep_draft_logits else None) for b in range(B)]

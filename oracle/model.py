@@ -144,13 +144,14 @@ class Transformer:
     def new_cache(self) -> KVCache:
         return KVCache(self.shape.n_layers)
 
-    def forward(self, seqs: Sequence[Tuple[KVCache, Sequence[int]]]):
+    def forward(self, seqs: Sequence[Tuple[KVCache, Sequence[int]]], last_only: bool = False):
         """Append each sequence's new tokens after its cache and run them through the model.
 
         seqs: list of (cache, tokens). Token i of a sequence sits at position len(cache) + i and
         attends to every cached position and to its own sequence's new tokens up to itself.
         Caches are extended in place. Returns (logits, hidden) lists, one [n_i, V] / [n_i, D]
-        pair per sequence; ``hidden`` is the final-normed state that feeds the LM head."""
+        pair per sequence; ``hidden`` is the final-normed state that feeds the LM head. With
+        ``last_only`` the LM head runs on each sequence's last row only ([1, V] / [1, D])."""
         S = self.shape
         H, KVH, hd = S.n_heads, S.n_kv_heads, S.head_dim
         G = H // KVH
@@ -178,18 +179,23 @@ class Transformer:
                 K = np.repeat(K, G, axis=1)      # [T, H, hd]: query head h reads kv head h // G
                 Vv = np.repeat(Vv, G, axis=1)
                 T = K.shape[0]
-                scores = np.einsum("ihd,thd->hit", q[r0:r1], K) / np.sqrt(hd)
                 n = r1 - r0
                 visible = starts[s] + np.arange(n)[:, None] + 1   # row i sees positions < visible
                 mask = np.arange(T)[None, :] >= visible           # [n, T]
-                scores = np.where(mask[None, :, :], -np.inf, scores)
-                p = softmax(scores, axis=-1)
-                att[r0:r1] = np.einsum("hit,thd->ihd", p, Vv)
+                qh = q[r0:r1].transpose(1, 0, 2)                  # [H, n, hd]
+                for h0 in range(0, H, G):                         # one KV head's query heads
+                    sc = (qh[h0:h0 + G] @ K[:, h0:h0 + G].transpose(1, 2, 0)) / np.sqrt(hd)
+                    sc = np.where(mask[None, :, :], -np.inf, sc)  # [G, n, T]
+                    p = softmax(sc, axis=-1)
+                    att[r0:r1, h0:h0 + G] = (p @ Vv[:, h0:h0 + G].transpose(1, 0, 2)).transpose(1, 0, 2)
             h = h + att.reshape(N, H * hd) @ self.w(f"l{l}.wo").T
             a = rms_norm(h, self.w(f"l{l}.ffn_norm"), S.norm_eps)
             g = a @ self.w(f"l{l}.w_gate").T
             u = a @ self.w(f"l{l}.w_up").T
             h = h + (silu(g) * u) @ self.w(f"l{l}.w_down").T
+        if last_only:
+            h = h[offs[1:] - 1]
+            offs = np.arange(len(seqs) + 1)
         hf = rms_norm(h, self.w("final_norm"), S.norm_eps)
         logits = hf @ self.w("lm_head").T
         return ([logits[offs[s]:offs[s + 1]] for s in range(len(seqs))],

@@ -148,7 +148,7 @@ int check_run(const cdsl_run_cfg* r, int vocab, std::string* why) {
   if (r->d < 1 || r->d > 16) return bad("d must be in 1..16");
   if (r->max_prompt < 1 || r->max_new < 1) return bad("max_prompt and max_new must be >= 1");
   if ((long long)r->max_prompt + r->max_new > (long long)(attn_max_chunks() - 1) * attn_chunk())
-    return bad("max_prompt + max_new exceeds the attention limit (4032 positions)");
+    return bad("max_prompt + max_new exceeds the attention limit (8128 positions)");
   if (r->n_keywords < 1 || r->n_keywords > 32) return bad("n_keywords must be in 1..32");
   const int ps = r->page_size ? r->page_size : 64;
   if (ps < 16 || ps > 256 || (ps & (ps - 1))) return bad("page_size must be a power of two in 16..256");

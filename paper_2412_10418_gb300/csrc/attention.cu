@@ -31,7 +31,7 @@ namespace cg = cooperative_groups;
 
 constexpr int ACH = 64;              // key slots per chunk
 constexpr int AQB = 40;              // query vectors per cluster (at most)
-constexpr int MAXP = 64;             // chunks (prefix + tail) of a pass
+constexpr int MAXP = 128;            // chunks (prefix + tail) of a pass
 constexpr int ACL = 16;              // blocks per cluster (at most)
 constexpr int MAXCB = MAXP / 8;      // chunks per block (at most; clusters have >= 8 blocks
                                      // whenever a pass has more than 8 chunks)
@@ -63,7 +63,8 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   __shared__ int s_wcnt[AWARPS];
   __shared__ int s_nrows, s_maxnp;
   __shared__ float s_pm[QB], s_pl[QB];          // the block's partial (m, l) per query vector
-  __shared__ const float* s_kp[MAXCB * ACH];    // K row of every key slot of the block's chunks
+  __shared__ int s_kslot[MAXCB * ACH];          // every key slot of the block's chunks: the page
+                                                // (prefix chunk) or tail row (tail chunk), -1 empty
   __shared__ int s_ktb[MAXCB * ACH];            // tail slots: tail base of the beam,
   __shared__ uint8_t s_kj[MAXCB * ACH];         //   index in it
 
@@ -88,7 +89,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   //      kernel), the committed page table and the tail layout come from kernels the launch
   //      chain has already completed, so everything up to the key slots precedes the wait.
   if (threadIdx.x < QB) s_row[threadIdx.x] = -1;
-  for (int i = threadIdx.x; i < MAXCB * ACH; i += ATHREADS) s_kp[i] = nullptr;
+  for (int i = threadIdx.x; i < MAXCB * ACH; i += ATHREADS) s_kslot[i] = -1;
   if (threadIdx.x == 0) s_nrows = 0;
   __syncthreads();
   for (int base = 0; base < a.R; base += ATHREADS) {
@@ -167,16 +168,13 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     if (c < n_p) {   // prefix positions c*64 .. c*64 + 63 below the longest prefix
       const int t = c * ACH + (threadIdx.x & (ACH - 1));
       if (threadIdx.x < ACH && t < maxnp) {
-        const int page = a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)];
-        if (page >= 0)
-          s_kp[i * ACH + threadIdx.x] = a.kv.pool + kv_prefix_offset(a.kv, a.layer, page, 0, g,
-                                                                     t & ((1 << a.kv.page_shift) - 1));
+        s_kslot[i * ACH + threadIdx.x] = a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)];
       }
     } else if (warp == 0) {   // tail slots [lo, lo + 64) of the concatenation
       const int lo = (c - n_p) * ACH, off = s_toff[lane], len = s_tlen[lane], tb = s_ttb[lane];
       for (int e = max(0, lo - off); e < len && off + e < lo + ACH; ++e) {
         const int sl = i * ACH + off + e - lo;
-        s_kp[sl] = a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, tb + e, g);
+        s_kslot[sl] = tb + e;
         s_ktb[sl] = tb;
         s_kj[sl] = (uint8_t)e;
       }
@@ -225,9 +223,12 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     for (int u = 0; u < PER; ++u) {
       const int idx = threadIdx.x + u * ATHREADS;
       const int j = idx / (HD / 4), e4 = idx % (HD / 4);
-      const float* kp = s_kp[i * ACH + j];
+      const int ks = s_kslot[i * ACH + j];
       kr[u] = vr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (kp) {
+      if (ks >= 0) {
+        const float* kp = tail ? a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, ks, g)
+                               : a.kv.pool + kv_prefix_offset(a.kv, a.layer, ks, 0, g,
+                                                              (t0 + j) & ((1 << a.kv.page_shift) - 1));
         kr[u] = __ldg(reinterpret_cast<const float4*>(kp + 4 * e4));
         vr[u] = __ldg(reinterpret_cast<const float4*>(kp + v_delta + 4 * e4));
       }
@@ -283,8 +284,8 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
       } else {                    // tail: the row's own beam, causal within it
         const int tb = s_tb[qi], nt = s_nt[qi];
         const int k0 = i * ACH + lane, k1 = k0 + 32;
-        ok0 = s_kp[k0] && s_ktb[k0] == tb && s_kj[k0] < nt;
-        ok1 = s_kp[k1] && s_ktb[k1] == tb && s_kj[k1] < nt;
+        ok0 = s_kslot[k0] >= 0 && s_ktb[k0] == tb && s_kj[k0] < nt;
+        ok1 = s_kslot[k1] >= 0 && s_ktb[k1] == tb && s_kj[k1] < nt;
       }
       const float a0 = ok0 ? s[q][0] : -INFINITY, a1 = ok1 ? s[q][1] : -INFINITY;
       const float m_new = fmaxf(m_run[q], warp_max(fmaxf(a0, a1)));

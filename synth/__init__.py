@@ -136,8 +136,17 @@ SEVEN_B_SLICE = Workload(
     batch=1, prompt_len=512, prompt_dist="zipf", k=4, d=4, max_new=128, n_keywords=5,
     reward_head=True)
 
+# Two layers of each 13B-shaped model, in the 13B launch configuration (4 prompts of 1024
+# tokens, k = 8, d = 6: 224 verify rows): full-size parity checks.
+THIRTEEN_B_SLICE = Workload(
+    name="13b-2layer-bf16", dtype=DTYPE_BF16,
+    target=dataclasses.replace(THIRTEEN_B.target, n_layers=2),
+    draft=dataclasses.replace(DRAFT_1B, n_layers=2),
+    batch=4, prompt_len=1024, prompt_dist="zipf", k=8, d=6, max_new=256, n_keywords=5,
+    reward_head=True)
+
 WORKLOADS: Dict[str, Workload] = {w.name: w for w in (TINY, SMALL, SEVEN_B, THIRTEEN_B,
-                                                      SEVEN_B_SLICE)}
+                                                      SEVEN_B_SLICE, THIRTEEN_B_SLICE)}
 
 
 def scaled(w: Workload, **changes) -> Workload:

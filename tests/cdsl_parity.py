@@ -60,10 +60,11 @@ def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0, accepta
     return eng
 
 
-def oracle_models(s: Setup):
+def oracle_models(s: Setup, keep_widened=True):
     wl = s.wl
-    tgt = oracle.Transformer(wl.target, s.t_host)
-    drf = tgt if s.d_host is s.t_host else oracle.Transformer(wl.draft, s.d_host)
+    tgt = oracle.Transformer(wl.target, s.t_host, keep_widened=keep_widened)
+    drf = tgt if s.d_host is s.t_host else oracle.Transformer(wl.draft, s.d_host,
+                                                              keep_widened=keep_widened)
     return tgt, drf
 
 
@@ -132,11 +133,11 @@ def decider_from(g, tol, tol_r):
 
 
 def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_size=16,
-               max_chunk=0, acceptance=0, seed=0):
+               max_chunk=0, acceptance=0, seed=0, torch_weights=None, keep_widened=True):
     """Step the GPU and the oracle together; every step is compared element by element."""
-    eng = eng or make_engine(s, page_size=page_size, max_chunk=max_chunk, acceptance=acceptance,
-                             seed=seed)
-    tgt, drf = oracle_models(s)
+    eng = eng or make_engine(s, torch_weights=torch_weights, page_size=page_size,
+                             max_chunk=max_chunk, acceptance=acceptance, seed=seed)
+    tgt, drf = oracle_models(s, keep_widened)
     states = oracle_prefill(s, tgt, drf)
     run = run_params(s.wl, acceptance, seed)
     report: Dict[str, float] = {}
