@@ -43,6 +43,9 @@ def parse():
     ap.add_argument("--decoder", choices=["cdsl", "cdlh"], default="cdsl",
                     help="cdlh: the lookaheads come from M_p itself and no lookahead is ever "
                          "accepted (Alg. 2 CDLH on the same kernels)")
+    ap.add_argument("--verify-sweep", action="store_true",
+                    help="time one cdsl_verify + cdsl_select per (k, d, prefix) point of the "
+                         "7B-shape verify sweep instead of the step benchmark")
     ap.add_argument("--oracle-layers", type=int, default=2,
                     help="target layers the oracle sample runs (scaled to the full depth)")
     return ap.parse_args()
@@ -469,9 +472,73 @@ def reference_main(args):
     print(json.dumps(out), flush=True)
 
 
+def verify_sweep(args):
+    """The verify-kernel sweep on the 7B-shape target: for k in {2,4,8,16}, d in {2,...,10},
+    prefix in {512,...,4096}, one cdsl_verify + cdsl_select call (after an untimed lookahead)
+    timed with CUDA events on the engine's stream (median of 3 after 1 warm-up), next to k*d
+    sequential target decode steps (the k=1, d=1 verify of the same prefix, 2 rows, stands in
+    for one decode step). One JSON line per point."""
+    import torch
+    import synth
+    import paper_2412_10418_gb300 as cdsl
+    from paper_2412_10418_gb300 import build as b
+    b.build()
+    wl0 = workload("7b-bf16")
+    tw = synth.model_weights(wl0, "target", device="cuda")
+    dw = synth.model_weights(wl0, "draft", device="cuda")
+    head = torch.from_numpy(synth.reward_head(wl0)).cuda()
+    wbytes = wl0.target.n_params() * 2
+    pk = peaks()
+    hbm = pk["hbm_gbs"] if pk else 6800.0
+    tfl = pk.get("bf16_tflops") if pk else None
+
+    def time_point(k, d, prefix, reps=3):
+        wl = synth.scaled(wl0, k=k, d=d, prompt_len=prefix, max_new=4 * reps + 8)
+        eng = cdsl.Engine(wl.target, wl.draft, wl.dtype,
+                          [tw[n] for n, _ in wl.target.weight_specs()],
+                          [dw[n] for n, _ in wl.draft.weight_specs()], batch=1, k=k, d=d,
+                          max_prompt=prefix, max_new=wl.max_new, n_keywords=wl.n_keywords,
+                          a_t=wl.a_t, r_t=wl.r_t, reward_head=head, device="cuda")
+        prefill(eng, wl)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ts = []
+        for r in range(reps + 1):
+            eng.lookahead()
+            eng.stream.synchronize()
+            e0.record(eng.stream)
+            eng.verify()
+            eng.select()
+            e1.record(eng.stream)
+            e1.synchronize()
+            if r:
+                ts.append(e0.elapsed_time(e1) * 1000.0)
+        eng.close()
+        return sorted(ts)[len(ts) // 2]
+
+    for prefix in (512, 1024, 2048, 4096):
+        t_dec = time_point(1, 1, prefix)
+        for k in (2, 4, 8, 16):
+            for d in (2, 4, 6, 8, 10):
+                us = time_point(k, d, prefix)
+                rows = k * (d + 1)
+                flops = 2.0 * wl0.target.n_params() * rows
+                out = {"sweep": "verify", "k": k, "d": d, "prefix": prefix, "rows": rows,
+                       "verify_select_us": round(us, 1),
+                       "weights_gbs": round(wbytes / (us * 1e-6) / 1e9, 1),
+                       "hbm_frac": round(wbytes / (us * 1e-6) / 1e9 / hbm, 3),
+                       "tflops": round(flops / (us * 1e-6) / 1e12, 2),
+                       "tensor_frac": round(flops / (us * 1e-6) / 1e12 / tfl, 4) if tfl else None,
+                       "decode_step_us": round(t_dec, 1),
+                       "sequential_kd_decode_us": round(k * d * t_dec, 1),
+                       "speedup_vs_sequential": round(k * d * t_dec / us, 2)}
+                print(json.dumps(out), flush=True)
+
+
 if __name__ == "__main__":
     a = parse()
     if a.impl == "reference":
         reference_main(a)
+    elif a.verify_sweep:
+        verify_sweep(a)
     else:
         gpu_main(a)

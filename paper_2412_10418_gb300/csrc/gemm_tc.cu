@@ -437,10 +437,12 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   // placed whole within a GPC; on 152 SMs at two blocks each, grids of clusters past ~87 % of
   // the block slots no longer fit in one wave (measured), hence the cap.
   const int cap = per_sm * n_sm * 87 / 100;
+  // (the whole partial tile, n_pad rows, stays in shared memory: two stages must still fit)
+  const bool tile_fits = fit(budget, p.n_pad) >= 2;
   int S = cluster;
-  if (S < 0) S = (p.n_pad <= kEpRowsMax && 2 * p.tiles <= cap) ? std::min(8, cap / p.tiles) : 0;
+  if (S < 0) S = (tile_fits && 2 * p.tiles <= cap) ? std::min(8, cap / p.tiles) : 0;
   S = std::min(std::min(S, p.kb_total), g_max_cluster);
-  if (S >= 2 && p.n_pad <= kEpRowsMax) {
+  if (S >= 2 && tile_fits) {
     p.cluster = S;
     p.ctas = p.tiles * S;
     p.ep_rows = p.n_pad;   // the whole partial tile stays in shared memory
