@@ -204,6 +204,17 @@ def reward(keywords, generated: Sequence[int], h_last: np.ndarray, w_head: np.nd
     return 0.5 * cov + 0.5 / (1.0 + np.exp(-z))
 
 
+def runtime_per_token(c: float, draft_calls: float, target_calls: float) -> float:
+    """Sec. 4.3 runtime model: P = c * (M_q calls per token) + (M_p calls per token), where c is
+    the cost of one M_q call in units of one M_p call (the ratio of their greedy tokens/s)."""
+    return c * draft_calls + target_calls
+
+
+def speedup(p_base: float, p_method: float) -> float:
+    """Sec. 4.3: the speedup of a method over a baseline is the ratio of their runtimes P."""
+    return p_base / p_method
+
+
 # ------------------------------------------------------------------------------------------
 # Per-prompt decoding state
 # ------------------------------------------------------------------------------------------

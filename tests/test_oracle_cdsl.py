@@ -354,3 +354,25 @@ def test_speculative_vs_hard_on_different_models():
                     u = oracle.uniform24(run.seed, oracle.draw_index(step, 1, 0, run.k, i, run.d, j))
                     ratio = np.exp(rec.logp[i, j] - rec.logq[i, j])
                     assert (u <= ratio) == (j < rec.n[i])
+
+
+# ---------------------------------------------------------------- Sec. 4.3 cost model
+
+def test_cost_model_reproduces_tables_5_and_6():
+    """Speedup over CDLH from c (Table 5) and the calls per token (Table 6): P = c * draft
+    calls + target calls, CDLH's P = its target calls; every printed speedup is reproduced
+    within what the printed inputs' rounding allows (2 decimals for calls, 3 for c, 2 for the
+    speedup)."""
+    n = 0
+    for line in open(os.path.join(GOLDEN, "cost_model_tables.txt")):
+        if line.startswith("#") or not line.strip():
+            continue
+        f = line.split()
+        c, dc, tc, cdlh, printed = map(float, f[3:8])
+        p = oracle.runtime_per_token(c, dc, tc)
+        got = oracle.speedup(oracle.runtime_per_token(c, 0.0, cdlh), p)
+        dp = 0.0005 * dc + c * 0.005 + 0.005
+        bound = got * (dp / p + 0.005 / cdlh) + 0.005
+        assert abs(got - printed) <= bound, (f[:3], got, printed, bound)
+        n += 1
+    assert n == 14
