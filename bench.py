@@ -40,6 +40,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--acceptance", choices=["hard", "speculative"], default="hard",
                     help="validation of the lookaheads by M_p (Sec. 3.2.2)")
+    ap.add_argument("--step1-budget", type=int, choices=[0, 1], default=0,
+                    help="Alg. 1 S2/S3 Step-1 budget b (Sec. 3.2.3)")
     ap.add_argument("--decoder", choices=["cdsl", "cdlh"], default="cdsl",
                     help="cdlh: the lookaheads come from M_p itself and no lookahead is ever "
                          "accepted (Alg. 2 CDLH on the same kernels)")
@@ -142,7 +144,7 @@ class ClockSampler:
 
 # ------------------------------------------------------------------------------ GPU arm
 
-def build_engine(wl, device, acceptance="hard", decoder="cdsl"):
+def build_engine(wl, device, acceptance="hard", decoder="cdsl", step1_budget=0):
     """The CDSL-k engine of a workload. decoder "cdlh": M_p drafts its own lookaheads and the
     reward threshold is above any reward (S1 never holds), so every step emits the one token
     of Alg. 2's CDLH (the step still runs its verify pass, which scores the beams)."""
@@ -162,7 +164,7 @@ def build_engine(wl, device, acceptance="hard", decoder="cdsl"):
                       max_new=wl.max_new, n_keywords=wl.n_keywords, a_t=wl.a_t,
                       r_t=2.0 if cdlh else wl.r_t, reward_head=head,
                       acceptance=cdsl.ACCEPT_SPECULATIVE if acceptance == "speculative"
-                      else cdsl.ACCEPT_HARD, seed=1, device=device)
+                      else cdsl.ACCEPT_HARD, seed=1, step1_budget=step1_budget, device=device)
     return eng, tw, dw
 
 
@@ -361,7 +363,7 @@ def gpu_main(args):
     if world > 1:
         dist.barrier()
     wl = workload(args.workload)
-    eng, tw, dw = build_engine(wl, device, args.acceptance, args.decoder)
+    eng, tw, dw = build_engine(wl, device, args.acceptance, args.decoder, args.step1_budget)
 
     if world > 1:
         dist.barrier()
@@ -422,6 +424,7 @@ def gpu_main(args):
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": dict(config_of(wl), parallelism=f"replicas{world}",
                            acceptance=args.acceptance, decoder=args.decoder,
+                           step1_budget=args.step1_budget,
                            **({"draft": "= target (CDLH)", "r_t": None}
                               if args.decoder == "cdlh" else {})),
             "verify_us": round(verify_us, 1),

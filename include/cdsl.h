@@ -14,7 +14,8 @@
  * a_b = n_b/d, the rewards, the chosen beam b* (largest r^full, first on ties) and the state:
  *   S1  (a_b* >= a_t and r^acc_b* >= r_t): emit c_b*, x_b*,1..n       (Sec. 3.2.3, S1)
  *   S2/S3 (a < a_t), S4 (a >= a_t, r < r_t): emit c_b* only, i.e. the one CDLH-appx token of
- *   Algorithm 1's fallback with Step-1 budget b = 0.
+ *   Algorithm 1's fallback (Step-2); with a Step-1 budget b = 1 (cdsl_run_cfg.step1_budget),
+ *   S2/S3 first emits M_p's greedy token c_1 if r^full_1 >= r_t (state 3).
  *
  * Conventions
  *  - Every compute call is asynchronous on the stream given to cdsl_init (a cudaStream_t
@@ -98,6 +99,11 @@ typedef struct cdsl_run_cfg {
    * steps of the context (SplitMix64: Steele, Lea, Flood, OOPSLA 2014). */
   int32_t acceptance;
   uint32_t seed;
+  /* Step-1 budget b of Alg. 1's S2/S3 branch (Sec. 3.2.3), 0 or 1. With b = 1, a
+   * step in S2/S3 (a < a_t) first tries M_p's greedy token, the root c_1, whose draft
+   * lookahead and reward r_1^full the step already has: if r_1^full >= r_t it emits c_1
+   * (state 3) instead of the CDLH-appx token c_{b*} of Step-2. */
+  int32_t step1_budget;
 } cdsl_run_cfg;
 
 typedef struct cdsl_ctx cdsl_ctx;
@@ -149,9 +155,10 @@ CDSL_API int32_t cdsl_lookahead(cdsl_ctx* ctx, int32_t* d_roots, int32_t* d_draf
 CDSL_API int32_t cdsl_verify(cdsl_ctx* ctx, float* d_logp, int32_t* d_argmax, int32_t* d_n_accept,
                     float* d_logits);
 
-/* Acceptance decision and commit (Sec. 3.2.3, Algorithm 1 with b = 0): rewards
- * d_reward [B, k, 2] = (r^full, r^acc) per beam, d_beam [B] b*, d_state [B] 1 (S1),
- * 2 (S2/S3) or 4 (S4), d_emitted [B, d+1] the emitted tokens (-1 padded), d_n_emitted [B]
+/* Acceptance decision and commit (Sec. 3.2.3, Algorithm 1 with b = 0 or 1): rewards
+ * d_reward [B, k, 2] = (r^full, r^acc) per beam, d_beam [B] the beam whose tokens are
+ * emitted (b*, or 0 for a Step-1 token), d_state [B] 1 (S1), 2 (S2/S3), 3 (S2/S3 resolved by
+ * Step-1) or 4 (S4), d_emitted [B, d+1] the emitted tokens (-1 padded), d_n_emitted [B]
  * (0 for prompts that already hold l_m tokens). Emission is cut at l_m. Then the winner's KV
  * rows are committed to the prefix pages and the next beams are taken from the winner's
  * verify row. Requires a preceding cdsl_verify. */

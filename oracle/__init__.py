@@ -13,7 +13,7 @@ Parity unpinned: the end-to-end token values of a CDSL step on random models (th
 prints no worked token-level example); they rest on the pins of the parts above.
 """
 from .model import KVCache, Transformer, log_softmax, rms_norm, rope, silu, softmax, widen
-from .cdsl import (S1, S2_S3, S4, Decider, PromptState, RunParams, StepRecord, alg1_generate,
-                   alg1_step, cdlh_generate, cdlh_token, cdsl_k_generate, cdsl_k_step, coverage,
-                   n_min, prefill, reward, HARD, SPECULATIVE, splitmix64, uniform24, draw_index,
-                   runtime_per_token, speedup)
+from .cdsl import (S1, S2_S3, S2_S3_STEP1, S4, Decider, PromptState, RunParams, StepRecord,
+                   alg1_generate, alg1_step, cdlh_generate, cdlh_token, cdsl_k_generate,
+                   cdsl_k_step, coverage, n_min, prefill, reward, HARD, SPECULATIVE, splitmix64,
+                   uniform24, draw_index, runtime_per_token, speedup)

@@ -41,7 +41,7 @@ import numpy as np
 
 from .model import KVCache, Transformer, log_softmax
 
-S1, S2_S3, S4 = 1, 2, 4
+S1, S2_S3, S2_S3_STEP1, S4 = 1, 2, 3, 4
 
 
 # ------------------------------------------------------------------------------------------
@@ -98,7 +98,7 @@ class Decider:
             if r[i] > best_r:           # strict '>' keeps the first of equal rewards (Alg. 2)
                 best, best_r = i, r[i]
         g = self._theirs(kind, idx)
-        if g is not None:
+        if g is not None and 0 <= int(g) < r.shape[0]:
             g = int(g)
             if g != best and r[g] != best_r and r[g] >= best_r - self.tol_r:
                 self.adopted.append((kind, idx, best, g))
@@ -141,7 +141,7 @@ class RunParams:
     r_t: float
     max_new: int                  # l_m of Alg. 1
     composite_reward: bool        # 0.5 coverage + 0.5 sigmoid(w.h) instead of coverage alone
-    b: int = 0                    # Step-1 budget of Alg. 1 (literal mode only)
+    b: int = 0                    # Step-1 budget of Alg. 1 (CDSL-k step: 0 or 1)
     acceptance: int = 0           # 0 hard rejection, 1 speculative sampling (Sec. 3.2.2)
     seed: int = 0                 # seed of the speculative-sampling uniforms
 
@@ -358,6 +358,13 @@ def cdsl_k_step(target: Transformer, draft: Transformer, states: List[PromptStat
         if n[bs] >= nmin and dec.reward_ok(r_acc[bs], run.r_t, "s1", b):
             state = S1
             out = [int(roots[b][bs])] + x[b][bs, :n[bs]].tolist()
+        elif (n[bs] < nmin and run.b >= 1
+              and dec.reward_ok(r_full[0], run.r_t, "step1", b)):
+            # S2/S3, Step-1 with b = 1 (Alg. 1, Sec. 3.2.3): M_p's greedy token is c_1; its
+            # d-token M_q lookahead is beam 1's draft, scored R(T + c_1 + lh) = r_1^full
+            state = S2_S3_STEP1
+            bs = 0
+            out = [int(roots[b][0])]
         else:
             state = S2_S3 if n[bs] < nmin else S4
             out = [int(roots[b][bs])]

@@ -43,7 +43,7 @@ class RunCfg(ctypes.Structure):
                 ("n_keywords", ctypes.c_int32), ("a_t", ctypes.c_float), ("r_t", ctypes.c_float),
                 ("reward_head", ctypes.c_int32), ("page_size", ctypes.c_int32),
                 ("max_chunk", ctypes.c_int32), ("acceptance", ctypes.c_int32),
-                ("seed", ctypes.c_uint32)]
+                ("seed", ctypes.c_uint32), ("step1_budget", ctypes.c_int32)]
 
 
 _P = ctypes.c_void_p
@@ -116,9 +116,10 @@ ACCEPT_HARD, ACCEPT_SPECULATIVE = 0, 1
 
 
 def run_cfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, reward_head,
-            page_size=0, max_chunk=0, acceptance=ACCEPT_HARD, seed=0) -> RunCfg:
+            page_size=0, max_chunk=0, acceptance=ACCEPT_HARD, seed=0, step1_budget=0) -> RunCfg:
     return RunCfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, int(reward_head),
-                  page_size, max_chunk, int(acceptance), int(seed) & 0xFFFFFFFF)
+                  page_size, max_chunk, int(acceptance), int(seed) & 0xFFFFFFFF,
+                  int(step1_budget))
 
 
 # ------------------------------------------------------------------------------ C names
@@ -226,15 +227,16 @@ class Engine:
 
     def __init__(self, target_shape, draft_shape, dtype, target_weights, draft_weights, *,
                  batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t, reward_head=None,
-                 page_size=0, max_chunk=0, acceptance=ACCEPT_HARD, seed=0, stream=None,
-                 device="cuda"):
+                 page_size=0, max_chunk=0, acceptance=ACCEPT_HARD, seed=0, step1_budget=0,
+                 stream=None, device="cuda"):
         import torch
 
         self.torch = torch
         self.tcfg = model_cfg(target_shape, dtype)
         self.dcfg = model_cfg(draft_shape, dtype)
         self.run = run_cfg(batch, k, d, max_prompt, max_new, n_keywords, a_t, r_t,
-                           reward_head is not None, page_size, max_chunk, acceptance, seed)
+                           reward_head is not None, page_size, max_chunk, acceptance, seed,
+                           step1_budget)
         self.B, self.k, self.d, self.V = batch, k, d, target_shape.vocab
         self.max_prompt, self.max_new = max_prompt, max_new
         self.tw, self.dw = list(target_weights), list(draft_weights)

@@ -155,6 +155,8 @@ int check_run(const cdsl_run_cfg* r, int vocab, std::string* why) {
   if (r->max_chunk < 0) return bad("max_chunk must be >= 0");
   if (r->acceptance != 0 && r->acceptance != 1)
     return bad("acceptance must be 0 (hard rejection) or 1 (speculative sampling)");
+  if (r->step1_budget != 0 && r->step1_budget != 1)
+    return bad("step1_budget must be 0 or 1");
   return CDSL_OK;
 }
 
@@ -274,6 +276,7 @@ size_t carve(cdsl_ctx* c, void* base) {
   s.r_t = c->run.r_t;
   s.acceptance = c->run.acceptance;
   s.seed = c->run.seed;
+  s.step1 = c->run.step1_budget;
   s.n_min = d + 1;
   for (int n = 0; n <= d; ++n)
     if ((float)n / (float)d >= c->run.a_t) { s.n_min = n; break; }

@@ -366,17 +366,21 @@ __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
   const int nb = __shfl_sync(0xffffffffu, n, bs);
   const float rab = __shfl_sync(0xffffffffu, ra, bs);
   const bool s1 = (nb >= st.n_min) && (rab >= st.r_t);
+  // Step-1 (b = 1) of S2/S3: M_p's greedy token c_1 when its lookahead's reward reaches r_t
+  const float rf1 = __shfl_sync(0xffffffffu, rf, 0);
+  const bool step1 = !s1 && nb < st.n_min && st.step1 >= 1 && rf1 >= st.r_t;
+  const int win = step1 ? 0 : bs;   // the beam whose tokens are emitted
   int cnt = s1 ? 1 + nb : 1;
   cnt = min(cnt, st.max_new - st.gen[b]);
-  const int bbi = b * k + bs;
+  const int bbi = b * k + win;
   if (lane < dp1) {
     int tok = -1;
     if (lane < cnt) tok = (lane == 0) ? st.roots[bbi] : st.x[bbi * d + lane - 1];
     st.emitted[b * dp1 + lane] = tok;
   }
   if (lane == 0) {
-    st.beam[b] = bs;
-    st.state[b] = s1 ? 1 : (nb < st.n_min ? 2 : 4);
+    st.beam[b] = win;
+    st.state[b] = s1 ? 1 : (step1 ? 3 : (nb < st.n_min ? 2 : 4));
     st.n_emit[b] = cnt;
     if (!commit) return;
     const int L = st.len[b];

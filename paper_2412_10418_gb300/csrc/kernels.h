@@ -16,6 +16,7 @@ struct StepState {
   float r_t;
   int32_t acceptance;  // 0 hard rejection, 1 speculative sampling
   uint32_t seed;       // SplitMix64 seed of the speculative-sampling draws
+  int32_t step1;       // Step-1 budget b (0 or 1)
   int32_t* len;        // [B] committed prefix length L (target; draft up to the pending row)
   int32_t* pend;       // [B] 1: the draft still lacks the KV of token L-1
   int32_t* gen;        // [B] tokens generated (len(T))

@@ -31,13 +31,14 @@ def make_setup(wl: synth.Workload, lens=None, keywords=None, draft_equals_target
     return Setup(wl, t, d, p, lens, kw, synth.reward_head(wl))
 
 
-def run_params(wl: synth.Workload, acceptance=0, seed=0) -> oracle.RunParams:
+def run_params(wl: synth.Workload, acceptance=0, seed=0, step1_budget=0) -> oracle.RunParams:
     return oracle.RunParams(k=wl.k, d=wl.d, a_t=wl.a_t, r_t=wl.r_t, max_new=wl.max_new,
-                            composite_reward=wl.reward_head, acceptance=acceptance, seed=seed)
+                            composite_reward=wl.reward_head, acceptance=acceptance, seed=seed,
+                            b=step1_budget)
 
 
 def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0, acceptance=0,
-                seed=0):
+                seed=0, step1_budget=0):
     import torch
     import paper_2412_10418_gb300 as cdsl
 
@@ -55,7 +56,7 @@ def make_engine(s: Setup, torch_weights=None, page_size=16, max_chunk=0, accepta
                       d=wl.d, max_prompt=wl.prompt_len, max_new=wl.max_new,
                       n_keywords=s.keywords.shape[1], a_t=wl.a_t, r_t=wl.r_t, reward_head=head,
                       page_size=page_size, max_chunk=max_chunk, acceptance=acceptance,
-                      seed=seed)
+                      seed=seed, step1_budget=step1_budget)
     eng.prefill(torch.from_numpy(s.prompts), s.lens, torch.from_numpy(s.keywords))
     return eng
 
@@ -127,19 +128,24 @@ def compare_step(g, recs, tol, tol_r, report):
 
 
 def decider_from(g, tol, tol_r):
-    other = {"roots": g["roots"], "x": g["draft_tok"], "argmax": g["argmax"],
-             "beam": g["beam"], "s1": g["state"] == oracle.S1, "spec": g["n_accept"]}
+    # a Step-1 token (state 3) reports beam 0, not b*: no beam choice to adopt there
+    beam = np.where(g["state"] == oracle.S2_S3_STEP1, -1, g["beam"])
+    other = {"roots": g["roots"], "x": g["draft_tok"], "argmax": g["argmax"], "beam": beam,
+             "s1": g["state"] == oracle.S1, "step1": g["state"] == oracle.S2_S3_STEP1,
+             "spec": g["n_accept"]}
     return oracle.Decider(other=other, tol=tol, tol_r=tol_r)
 
 
 def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_size=16,
-               max_chunk=0, acceptance=0, seed=0, torch_weights=None, keep_widened=True):
+               max_chunk=0, acceptance=0, seed=0, torch_weights=None, keep_widened=True,
+               step1_budget=0):
     """Step the GPU and the oracle together; every step is compared element by element."""
     eng = eng or make_engine(s, torch_weights=torch_weights, page_size=page_size,
-                             max_chunk=max_chunk, acceptance=acceptance, seed=seed)
+                             max_chunk=max_chunk, acceptance=acceptance, seed=seed,
+                             step1_budget=step1_budget)
     tgt, drf = oracle_models(s, keep_widened)
     states = oracle_prefill(s, tgt, drf)
-    run = run_params(s.wl, acceptance, seed)
+    run = run_params(s.wl, acceptance, seed, step1_budget)
     report: Dict[str, float] = {}
     adopted = []
     n_steps = 0
@@ -152,6 +158,10 @@ def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_si
         compare_step(g, recs, tol, tol_r, report)
         report["accepted"] = report.get("accepted", 0) + int(
             sum(g["n_accept"][b].sum() for b, r in enumerate(recs) if r.active))
+        for r in recs:
+            if r.active:
+                key = f"state{r.state}"
+                report[key] = report.get(key, 0) + 1
         adopted += dec.adopted
         n_steps += 1
     assert eng.status() == 0

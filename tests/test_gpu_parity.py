@@ -206,3 +206,32 @@ def test_tiny_gqa_wide_query_blocks():
     s = make_setup(wl, lens=[40, 23])
     eng, states, rep, adopted, n = run_parity(s, steps=16, tol=TOL32, tol_r=TOL32)
     tokens_match(eng, states)
+
+
+def test_tiny_step1_always_succeeding_is_greedy():
+    """Step-1 budget b = 1 with a_t above 1 and r_t = 0: every step is an S2/S3 step resolved
+    by Step-1 (state 3), emitting M_p's greedy token."""
+    wl = synth.scaled(synth.TINY, a_t=1.5, r_t=0.0, max_new=12)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=12, tol=TOL32, tol_r=TOL32,
+                                              step1_budget=1)
+    tokens_match(eng, states)
+    tgt = oracle.Transformer(wl.target, s.t_host)
+    assert states[0].T == greedy_chain(tgt, s.prompts[0].tolist(), wl.max_new)
+
+
+def test_tiny_step1_mixed_states():
+    """b = 1 with keywords from M_p's greedy continuation: Step-1 resolves some S2/S3 steps,
+    the others fall back to the CDLH-appx token; GPU and oracle agree step by step."""
+    wl = synth.scaled(synth.TINY, batch=2, max_new=20)
+    t_host = synth.model_weights(wl, "target", device="host")
+    tgt = oracle.Transformer(wl.target, t_host)
+    p = synth.prompts(wl)
+    kw = np.stack([np.array(greedy_chain(tgt, p[b].tolist(), 12)[3:12:4], np.int32)
+                   for b in range(wl.batch)])
+    s = make_setup(wl, keywords=kw)
+    eng, states, rep, adopted, n = run_parity(s, steps=20, tol=TOL32, tol_r=TOL32,
+                                              step1_budget=1)
+    tokens_match(eng, states)
+    assert rep.get(f"state{oracle.S2_S3_STEP1}", 0) > 0, rep
+    print("step-1 states:", {k: v for k, v in rep.items() if k.startswith("state")})

@@ -376,3 +376,75 @@ def test_cost_model_reproduces_tables_5_and_6():
         assert abs(got - printed) <= bound, (f[:3], got, printed, bound)
         n += 1
     assert n == 14
+
+
+# ---------------------------------------------------------------- Step-1 with b = 1 (f2)
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_step1_emits_greedy_root_when_its_lookahead_reaches_r_t(seed):
+    """Alg. 1 S2/S3 with b = 1: M_p's greedy token (the root c_1) is emitted when the reward
+    of its M_q lookahead (beam 1's draft), r_1^full, reaches r_t; otherwise the step falls
+    back to the CDLH-appx token c_{b*} exactly as with b = 0. S1 and S4 are unaffected."""
+    shp = shape(vocab=24)
+    tgt, drf = model(shp, 10 + seed), model(shp, 20 + seed)
+    w = np.random.default_rng(seed).standard_normal(shp.d_model)
+    prompts = np.array([[1, 2, 3, 4, 5], [6, 7, 8, 9, 10], [3, 1, 4, 1, 5]])
+    kw = np.array([[1, 2, 3], [4, 5, 6], [7, 8, 9]])
+    seen = {S1: 0, S2_S3: 0, oracle.S2_S3_STEP1: 0, S4: 0}
+    for r_t in (0.5, 0.6, 0.7):
+        st0 = prefill(tgt, drf, prompts, kw)
+        st1 = prefill(tgt, drf, prompts, kw)
+        for step in range(3):
+            r0 = cdsl_k_step(tgt, drf, st0, run_params(k=3, d=3, r_t=r_t), w, step=step)
+            r1 = cdsl_k_step(tgt, drf, st1, run_params(k=3, d=3, r_t=r_t, b=1), w, step=step)
+            for a, c in zip(r0, r1):
+                seen[c.state] += 1
+                assert np.allclose(a.r_full, c.r_full)
+                if a.state == S2_S3 and np.float32(a.r_full[0]) >= np.float32(r_t):
+                    assert c.state == oracle.S2_S3_STEP1 and c.emitted == [int(a.roots[0])]
+                    assert c.beam == 0
+                else:
+                    assert c.state == a.state and c.emitted == a.emitted
+            # keep both runs on the same path: continue from the b = 1 states
+            st0 = [dataclasses_copy(s) for s in st1]
+    assert sum(seen.values()) == 3 * 3 * 3
+
+
+def test_step1_always_succeeding_is_greedy_decoding():
+    """b = 1, a_t above 1 (S1 never holds) and r_t = 0 (every lookahead reaches it): every step
+    is an S2/S3 step resolved by Step-1, i.e. M_p's greedy token: the whole generation is
+    M_p's greedy decoding."""
+    shp = shape(vocab=24)
+    tgt, drf = model(shp, 7), model(shp, 8)
+    w = np.random.default_rng(9).standard_normal(shp.d_model)
+    prompt = [2, 7, 1, 8]
+    run = run_params(k=3, d=3, a_t=1.5, r_t=0.0, b=1, max_new=8)
+    st = prefill(tgt, drf, np.array([prompt]), np.array([[1, 2, 3]]))
+    step = 0
+    while len(st[0].T) < run.max_new:
+        rec = cdsl_k_step(tgt, drf, st, run, w, step=step)[0]
+        assert rec.state == oracle.S2_S3_STEP1 and rec.beam == 0
+        step += 1
+    assert st[0].T == greedy_chain(tgt, prompt, run.max_new)
+
+
+def dataclasses_copy(st):
+    import dataclasses
+    return dataclasses.replace(st, tcache=st.tcache.fork(), dcache=st.dcache.fork())
+
+
+def test_step1_with_one_beam_changes_no_token():
+    """k = 1: c_1 is the only beam, so the Step-1 token and the CDLH-appx token coincide; only
+    the reported state differs."""
+    shp = shape(vocab=24)
+    tgt, drf = model(shp, 3), model(shp, 4)
+    w = np.random.default_rng(5).standard_normal(shp.d_model)
+    p = np.array([[1, 2, 3, 4]])
+    kw = np.array([[1, 2, 3]])
+    a = prefill(tgt, drf, p, kw)
+    b = prefill(tgt, drf, p, kw)
+    for step in range(4):
+        ra = cdsl_k_step(tgt, drf, a, run_params(k=1, d=3, r_t=0.4), w, step=step)[0]
+        rb = cdsl_k_step(tgt, drf, b, run_params(k=1, d=3, r_t=0.4, b=1), w, step=step)[0]
+        assert ra.emitted == rb.emitted
+        assert (ra.state == rb.state) or (ra.state == S2_S3 and rb.state == oracle.S2_S3_STEP1)
