@@ -42,9 +42,10 @@ def parse():
                     help="validation of the lookaheads by M_p (Sec. 3.2.2)")
     ap.add_argument("--step1-budget", type=int, choices=[0, 1], default=0,
                     help="Alg. 1 S2/S3 Step-1 budget b (Sec. 3.2.3)")
-    ap.add_argument("--decoder", choices=["cdsl", "cdlh"], default="cdsl",
+    ap.add_argument("--decoder", choices=["cdsl", "cdlh", "cdlh-appx"], default="cdsl",
                     help="cdlh: the lookaheads come from M_p itself and no lookahead is ever "
-                         "accepted (Alg. 2 CDLH on the same kernels)")
+                         "accepted (Alg. 2 CDLH on the same kernels); cdlh-appx: M_q's "
+                         "lookaheads, never accepted (Alg. 2 CDLH-appx)")
     ap.add_argument("--verify-sweep", action="store_true",
                     help="time one cdsl_verify + cdsl_select per (k, d, prefix) point of the "
                          "7B-shape verify sweep instead of the step benchmark")
@@ -147,7 +148,9 @@ class ClockSampler:
 def build_engine(wl, device, acceptance="hard", decoder="cdsl", step1_budget=0):
     """The CDSL-k engine of a workload. decoder "cdlh": M_p drafts its own lookaheads and the
     reward threshold is above any reward (S1 never holds), so every step emits the one token
-    of Alg. 2's CDLH (the step still runs its verify pass, which scores the beams)."""
+    of Alg. 2's CDLH (the step still runs its verify pass, which scores the beams).
+    "cdlh-appx": M_q's lookaheads, thresholds above any score: every step emits the one
+    CDLH-appx token c_{b*} (Alg. 2 with M_q as the lookahead model)."""
     import torch
     import synth
     import paper_2412_10418_gb300 as cdsl
@@ -161,8 +164,9 @@ def build_engine(wl, device, acceptance="hard", decoder="cdsl", step1_budget=0):
                       [tw[n] for n, _ in wl.target.weight_specs()],
                       [dw[n] for n, _ in dshape.weight_specs()],
                       batch=wl.batch, k=wl.k, d=wl.d, max_prompt=wl.prompt_len,
-                      max_new=wl.max_new, n_keywords=wl.n_keywords, a_t=wl.a_t,
-                      r_t=2.0 if cdlh else wl.r_t, reward_head=head,
+                      max_new=wl.max_new, n_keywords=wl.n_keywords,
+                      a_t=2.0 if decoder == "cdlh-appx" else wl.a_t,
+                      r_t=2.0 if decoder != "cdsl" else wl.r_t, reward_head=head,
                       acceptance=cdsl.ACCEPT_SPECULATIVE if acceptance == "speculative"
                       else cdsl.ACCEPT_HARD, seed=1, step1_budget=step1_budget, device=device)
     return eng, tw, dw
@@ -426,7 +430,8 @@ def gpu_main(args):
                            acceptance=args.acceptance, decoder=args.decoder,
                            step1_budget=args.step1_budget,
                            **({"draft": "= target (CDLH)", "r_t": None}
-                              if args.decoder == "cdlh" else {})),
+                              if args.decoder == "cdlh" else {}),
+                           **({"a_t": None, "r_t": None} if args.decoder == "cdlh-appx" else {})),
             "verify_us": round(verify_us, 1),
             "verify_gbs": round(verify_bytes / (verify_us * 1e-6) / 1e9, 1),
             "tokens_per_step": round(tokens_per_step, 3),

@@ -235,3 +235,21 @@ def test_tiny_step1_mixed_states():
     tokens_match(eng, states)
     assert rep.get(f"state{oracle.S2_S3_STEP1}", 0) > 0, rep
     print("step-1 states:", {k: v for k, v in rep.items() if k.startswith("state")})
+
+
+def test_tiny_cdlh_appx_on_the_same_kernels():
+    """Alg. 2 CDLH-appx on the GPU path: M_q's lookaheads are never accepted (a_t, r_t above
+    any score), so every step emits c_{b*}: the CDLH-appx token of the oracle's Alg. 2 with
+    M_q as the lookahead model, step by step and over the whole generation."""
+    wl = synth.scaled(synth.TINY, a_t=2.0, r_t=2.0, max_new=10)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=10, tol=TOL32, tol_r=TOL32)
+    assert n == wl.max_new
+    tokens_match(eng, states)
+    tgt = oracle.Transformer(wl.target, s.t_host)
+    drf = oracle.Transformer(wl.draft, s.d_host)
+    run = run_params(wl)
+    for b in range(wl.batch):
+        ref = oracle.cdlh_generate(tgt, drf, drf, s.prompts[b].tolist(), s.keywords[b].tolist(),
+                                   run, s.w_head)
+        assert states[b].T == ref.T
