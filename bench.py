@@ -225,7 +225,16 @@ def kernel_timing(eng, wl, n_steps):
     for _ in range(n_steps):
         eng.step()
     prof = {name: cdsl.cdsl_get_profile(eng.ctx, impl) for impl, name in cdsl.KERNEL_CLASSES.items()}
+    # tensor-core GEMM launches grouped by shape (equal algorithmic bytes = same projection)
+    groups = {}
+    for cls, ms, by, fl in cdsl.cdsl_get_profile_launches(eng.ctx):
+        if cls != 2:
+            continue
+        g = groups.setdefault(round(by), [0, 0.0])
+        g[0] += 1
+        g[1] += ms
     cdsl.cdsl_profile(eng.ctx, False)
+    prof["_gemm_shapes"] = groups
     # verify-step time: lookahead, then the verify call alone between events
     ts = []
     for _ in range(n_steps):
@@ -386,6 +395,7 @@ def gpu_main(args):
 
     n_prof = min(args.steps, 5)
     prof, verify_us = kernel_timing(eng, wl, n_prof)
+    shapes = prof.pop("_gemm_shapes")
     import paper_2412_10418_gb300 as cdsl
     gem = {k: v for k, v in prof.items() if k in cdsl.GEMM_IMPLS.values()}
     dom = max(gem.items(), key=lambda kv: kv[1]["ms"])
@@ -402,6 +412,12 @@ def gpu_main(args):
                 "launches_timed": dom[1]["launches"],
                 "avg_launch_us": round(dom[1]["ms"] * 1000.0 / max(1, dom[1]["launches"]), 2),
                 "bytes_per_launch": round(dom[1]["bytes"] / max(1, dom[1]["launches"]))}
+    # per projection shape (the same kernel, different launch shapes): the largest by time
+    by_shape = sorted(({"bytes_per_launch": b, "launches": n, "avg_us": round(ms * 1000.0 / n, 2),
+                        "GB/s": round(b / (ms / n / 1000.0) / 1e9, 1),
+                        "frac": round(b / (ms / n / 1000.0) / 1e9 / hbm, 3)}
+                       for b, (n, ms) in shapes.items()), key=lambda r: -r["avg_us"] * r["launches"])
+    roofline["by_shape"] = by_shape[:8]
     verify_bytes = (wl.target.n_params() * 2)
     e2e = None
     if not args.no_e2e:

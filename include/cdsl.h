@@ -195,6 +195,11 @@ CDSL_API int32_t cdsl_get_counters(cdsl_ctx* ctx, int64_t* h_counters);
  * or disabled timing (each call of cdsl_profile clears the record). */
 CDSL_API int32_t cdsl_profile(cdsl_ctx* ctx, int32_t enable);
 CDSL_API int32_t cdsl_get_profile(cdsl_ctx* ctx, int32_t impl, double* h_out);
+/* Per-launch form of the same record: for each of the first h_capacity recorded launches,
+ * in launch order, four doubles {class, milliseconds, algorithmic bytes, flops} at h_out
+ * [4 * i]; returns the number of records written (>= 0) or a negative status. Synchronizes
+ * the stream. */
+CDSL_API int32_t cdsl_get_profile_launches(cdsl_ctx* ctx, double* h_out, int32_t h_capacity);
 
 /* Synchronize the stream and return the device status word (a cdsl_status; CDSL_OK when no
  * device-side error was latched) in *h_device_status. Clears nothing. */

@@ -65,6 +65,7 @@ EXPORTS = {
     "cdsl_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_int32)]),
     "cdsl_profile": (_I, [_P, _I]),
     "cdsl_get_profile": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double)]),
+    "cdsl_get_profile_launches": (_I, [_P, ctypes.POINTER(ctypes.c_double), _I]),
     "cdsl_gemv_noalloc": (_I, [_P, _I, _I, _P, _I, _P, _P]),
     "cdsl_last_error": (ctypes.c_char_p, [_P]),
     "cdsl_destroy": (None, [_P]),
@@ -198,6 +199,15 @@ def cdsl_get_profile(ctx, impl: int):
     out = (ctypes.c_double * 4)()
     _check(lib().cdsl_get_profile(ctx, impl, out), ctx)
     return dict(launches=int(out[0]), ms=out[1], bytes=out[2], flops=out[3])
+
+
+def cdsl_get_profile_launches(ctx, capacity: int = 8192):
+    """Per-launch timing records [(class, ms, bytes, flops)] in launch order."""
+    out = (ctypes.c_double * (4 * capacity))()
+    n = lib().cdsl_get_profile_launches(ctx, out, capacity)
+    if n < 0:
+        raise CdslError(-n, cdsl_last_error(ctx))
+    return [(int(out[4 * i]), out[4 * i + 1], out[4 * i + 2], out[4 * i + 3]) for i in range(n)]
 
 
 def cdsl_gemv_noalloc(w, x, y, stream=None):

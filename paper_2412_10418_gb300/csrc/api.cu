@@ -899,6 +899,22 @@ int32_t cdsl_get_profile(cdsl_ctx* c, int32_t impl, double* h_out) {
   return cuda_check(c, "cdsl_get_profile");
 }
 
+int32_t cdsl_get_profile_launches(cdsl_ctx* c, double* h_out, int32_t h_capacity) {
+  if (!c || !h_out || h_capacity < 0) return -fail(c, CDSL_EINVAL, "ctx or out is NULL");
+  cudaError_t e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess)
+    return -fail(c, CDSL_ECUDA, std::string("cdsl_get_profile_launches: ") + cudaGetErrorString(e));
+  int32_t n = 0;
+  for (const auto& r : c->prof) {
+    if (n >= h_capacity) break;
+    float t = 0;
+    cudaEventElapsedTime(&t, c->ev_pool[r.ev], c->ev_pool[r.ev + 1]);
+    h_out[4 * n] = r.impl; h_out[4 * n + 1] = t; h_out[4 * n + 2] = r.bytes; h_out[4 * n + 3] = r.flops;
+    ++n;
+  }
+  return n;
+}
+
 int32_t cdsl_get_status(cdsl_ctx* c, int32_t* h_device_status) {
   if (!c || !h_device_status) return fail(c, CDSL_EINVAL, "ctx or status is NULL");
   int32_t v = 0;
