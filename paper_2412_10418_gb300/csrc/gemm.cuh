@@ -113,85 +113,107 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
     tid = threadIdx.x;
     nthr = blockDim.x;
   }
-  const int n_items = rt * 128;   // a multiple of 32: every warp sees 32 features of one row
-  for (int idx = tid; idx < n_items; idx += nthr) {
-    const int r = idx >> 7, v = idx & 127;
-    const int row = r0 + r;
-    const bool live = row < a.R;
-    float y = tile[r * ldt + v];
-    if (a.in_ss) y *= s_rs[r];
-    const int n = v0 + v;
-    switch (a.mode) {
-      case EPI_STORE:
-        if (live && n < a.n_virtual) a.out_f32[(size_t)row * a.ld_out + n] = y;
-        break;
-      case EPI_RESID: {
-        float hn = 0.f;
-        if (live && n < a.n_virtual) {
-          float* hp = a.out_f32 + (size_t)row * a.ld_out + n;
-          hn = *hp + y;
-          *hp = hn;
-          if (a.next_x)
-            store_act<T>(reinterpret_cast<T*>(a.next_x), a.act_plane, (size_t)row * a.ld_out + n,
-                         hn * to_f32<T>(reinterpret_cast<const T*>(a.next_g)[n]));
-        }
-        if (a.out_ss) {   // warp-uniform: 32 consecutive features of one row
-          const float sq = warp_sum(hn * hn);
-          float hw = 0.f;
-          if (a.head_w) {
-            const float gw = (live && n < a.n_virtual)
-                                 ? a.head_w[n] * to_f32<T>(reinterpret_cast<const T*>(a.next_g)[n])
-                                 : 0.f;
-            hw = warp_sum(gw * hn);
-          }
-          if ((v & 31) == 0 && live && n < a.n_virtual) {
-            a.out_ss[(size_t)(n >> 5) * a.ld_ss + row] = sq;
-            if (a.head_w) a.out_hw[(size_t)(n >> 5) * a.ld_ss + row] = hw;
-          }
-        }
-        break;
+  // Every field is read once, into registers, before the stores: `a` is reached through a
+  // reference (to the kernel parameter), which the compiler must otherwise assume the stores
+  // below may alias, re-reading it on every item.
+  const int mode = a.mode, R = a.R, nv = a.n_virtual;
+  const bool scaled = a.in_ss != nullptr;
+  const float* __restrict__ tl = tile;   // shared memory: never aliases the outputs
+  if (mode == EPI_STORE) {
+    float* __restrict__ const out = a.out_f32;
+    const size_t ld = (size_t)a.ld_out;
+    for (int idx = tid; idx < rt * 128; idx += nthr) {
+      const int r = idx >> 7, v = idx & 127, row = r0 + r, n = v0 + v;
+      float y = tl[r * ldt + v];
+      if (scaled) y *= s_rs[r];
+      if (row < R && n < nv) out[(size_t)row * ld + n] = y;
+    }
+  } else if (mode == EPI_RESID) {
+    float* __restrict__ const out = a.out_f32;
+    const size_t ld = (size_t)a.ld_out, plane = (size_t)a.act_plane, ld_ss = (size_t)a.ld_ss;
+    T* const next_x = reinterpret_cast<T*>(a.next_x);
+    const T* const next_g = reinterpret_cast<const T*>(a.next_g);
+    float* const out_ss = a.out_ss;
+    const float* const head_w = a.head_w;
+    float* const out_hw = a.out_hw;
+    // a multiple of 32 items per thread pass: every warp sees 32 features of one row
+    for (int idx = tid; idx < rt * 128; idx += nthr) {
+      const int r = idx >> 7, v = idx & 127, row = r0 + r, n = v0 + v;
+      const bool ok = row < R && n < nv;
+      float y = tl[r * ldt + v];
+      if (scaled) y *= s_rs[r];
+      float hn = 0.f;
+      if (ok) {
+        float* hp = out + (size_t)row * ld + n;
+        hn = *hp + y;
+        *hp = hn;
+        if (next_x)
+          store_act<T>(next_x, plane, (size_t)row * ld + n, hn * to_f32<T>(next_g[n]));
       }
-      case EPI_SWIGLU: {
-        if (!live || v >= 64) break;
-        const int f = (v0 >> 7) * 64 + v;
-        if (f >= a.d_ffn) break;
-        float u = tile[r * ldt + v + 64];
-        if (a.in_ss) u *= s_rs[r];
-        store_act<T>(reinterpret_cast<T*>(a.out_act), a.act_plane, (size_t)row * a.ld_act + f,
-                     silu_f(y) * u);
-        break;
+      if (out_ss) {   // warp-uniform
+        const float sq = warp_sum(hn * hn);
+        float hw = 0.f;
+        if (head_w) {
+          const float gw = ok ? head_w[n] * to_f32<T>(next_g[n]) : 0.f;
+          hw = warp_sum(gw * hn);
+        }
+        if ((v & 31) == 0 && ok) {
+          out_ss[(size_t)(n >> 5) * ld_ss + row] = sq;
+          if (head_w) out_hw[(size_t)(n >> 5) * ld_ss + row] = hw;
+        }
       }
-      case EPI_QKV: {
-        if (!live) break;
-        const int hd = a.kv.hd, half = hd >> 1;
-        const int nq = a.n_heads * hd, nk = a.kv.kvh * hd;
-        if (n >= nq + 2 * nk) break;
-        const RowDesc rd = a.rows[row];
-        float val = y;
-        const int e = n % hd;  // segments start on head boundaries
-        if (n < nq + nk) {     // q or k: rotate-half RoPE with the partner in this tile
-          const float2 cs = a.rope[(size_t)rd.pos * half + (e % half)];
-          float other = (e < half) ? tile[r * ldt + v + half] : tile[r * ldt + v - half];
-          if (a.in_ss) other *= s_rs[r];
-          val = (e < half) ? (y * cs.x - other * cs.y) : (y * cs.x + other * cs.y);
+    }
+  } else if (mode == EPI_SWIGLU) {
+    T* const out_act = reinterpret_cast<T*>(a.out_act);
+    const size_t ld_act = (size_t)a.ld_act, plane = (size_t)a.act_plane;
+    const int d_ffn = a.d_ffn, f0 = (v0 >> 7) * 64;
+    for (int idx = tid; idx < rt * 64; idx += nthr) {   // gate v, up v + 64
+      const int r = idx >> 6, v = idx & 63, row = r0 + r, f = f0 + v;
+      if (row >= R || f >= d_ffn) continue;
+      float g = tl[r * ldt + v], u = tl[r * ldt + v + 64];
+      if (scaled) {
+        g *= s_rs[r];
+        u *= s_rs[r];
+      }
+      store_act<T>(out_act, plane, (size_t)row * ld_act + f, silu_f(g) * u);
+    }
+  } else {   // EPI_QKV
+    const KvStore kv = a.kv;
+    float* const q_out = a.q_out;
+    const RowDesc* const rows = a.rows;
+    const float2* const rope = a.rope;
+    const int layer = a.layer;
+    const int hd = kv.hd, half = hd >> 1;
+    const int nq = a.n_heads * hd, nk = kv.kvh * hd;
+    for (int idx = tid; idx < rt * 128; idx += nthr) {
+      const int r = idx >> 7, v = idx & 127, row = r0 + r, n = v0 + v;
+      if (row >= R || n >= nq + 2 * nk) continue;
+      float y = tl[r * ldt + v];
+      if (scaled) y *= s_rs[r];
+      const RowDesc rd = rows[row];
+      float val = y;
+      const int e = n % hd;  // segments start on head boundaries
+      if (n < nq + nk) {     // q or k: rotate-half RoPE with the partner in this tile
+        const float2 cs = rope[(size_t)rd.pos * half + (e % half)];
+        float other = (e < half) ? tl[r * ldt + v + half] : tl[r * ldt + v - half];
+        if (scaled) other *= s_rs[r];
+        val = (e < half) ? (y * cs.x - other * cs.y) : (y * cs.x + other * cs.y);
+      }
+      if (n < nq) {
+        q_out[(size_t)row * nq + n] = val;
+      } else {
+        const int kvsel = (n < nq + nk) ? 0 : 1;
+        const int head = (n - nq - kvsel * nk) / hd;
+        float* dst = nullptr;
+        if (rd.kv_dst >= 0) {
+          dst = kv.tail + kv_tail_offset(kv, layer, kvsel, rd.kv_dst, head);
+        } else if (rd.kv_dst == KV_PREFIX) {
+          const int page = kv.page_table[rd.b * kv.max_pages + (rd.pos >> kv.page_shift)];
+          if (page >= 0)
+            dst = kv.pool + kv_prefix_offset(kv, layer, page, kvsel, head,
+                                             rd.pos & ((1 << kv.page_shift) - 1));
         }
-        if (n < nq) {
-          a.q_out[(size_t)row * nq + n] = val;
-        } else {
-          const int kvsel = (n < nq + nk) ? 0 : 1;
-          const int head = (n - nq - kvsel * nk) / hd;
-          float* dst = nullptr;
-          if (rd.kv_dst >= 0) {
-            dst = a.kv.tail + kv_tail_offset(a.kv, a.layer, kvsel, rd.kv_dst, head);
-          } else if (rd.kv_dst == KV_PREFIX) {
-            const int page = a.kv.page_table[rd.b * a.kv.max_pages + (rd.pos >> a.kv.page_shift)];
-            if (page >= 0)
-              dst = a.kv.pool + kv_prefix_offset(a.kv, a.layer, page, kvsel, head,
-                                                 rd.pos & ((1 << a.kv.page_shift) - 1));
-          }
-          if (dst) dst[e] = val;
-        }
-        break;
+        if (dst) dst[e] = val;
       }
     }
   }
@@ -199,18 +221,21 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
 
 __device__ __forceinline__ void input_row_scales(const GemmArgs& a, int r0, int n, float* rs,
                                                  int tid, int nthr) {
-  const int chunks = a.norm_D >> 5, items = n * 4;
+  const int D = a.norm_D, chunks = D >> 5, items = n * 4, R = a.R;
+  const float* const ss = a.in_ss;
+  const size_t ld = (size_t)a.ld_ss;
+  const float eps = a.norm_eps;
   for (int base = tid & ~31; base < items; base += nthr) {   // warp-uniform trip count
     const int idx = base + (tid & 31), r = idx >> 2, q = idx & 3, row = r0 + r;
-    const bool live = idx < items && row < a.R;
+    const bool live = idx < items && row < R;
     float acc = 0.f;
     if (live) {
 #pragma unroll 8
-      for (int c = q; c < chunks; c += 4) acc += a.in_ss[(size_t)c * a.ld_ss + row];
+      for (int c = q; c < chunks; c += 4) acc += ss[(size_t)c * ld + row];
     }
     acc += __shfl_xor_sync(0xffffffffu, acc, 1);   // (S_0 + S_1), (S_2 + S_3)
     acc += __shfl_xor_sync(0xffffffffu, acc, 2);   // (S_0 + S_1) + (S_2 + S_3)
-    if (idx < items && q == 0) rs[r] = live ? rsqrtf(acc / (float)a.norm_D + a.norm_eps) : 0.f;
+    if (idx < items && q == 0) rs[r] = live ? rsqrtf(acc / (float)D + eps) : 0.f;
   }
 }
 
