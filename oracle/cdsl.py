@@ -141,7 +141,7 @@ class RunParams:
     r_t: float
     max_new: int                  # l_m of Alg. 1
     composite_reward: bool        # 0.5 coverage + 0.5 sigmoid(w.h) instead of coverage alone
-    b: int = 0                    # Step-1 budget of Alg. 1 (CDSL-k step: 0 or 1)
+    b: int = 0                    # Step-1 budget of Alg. 1 (0 = Step-2 only)
     acceptance: int = 0           # 0 hard rejection, 1 speculative sampling (Sec. 3.2.2)
     seed: int = 0                 # seed of the speculative-sampling uniforms
 
@@ -269,6 +269,50 @@ class StepRecord:
     beam: int
     state: int
     emitted: List[int]
+    # Step-1 rounds after the first (budget b >= 2), in order: the round's M_p greedy token and
+    # its d-token M_q lookahead [tok, lh_1..lh_d], and the reward R(T + X + tok + lh)
+    step1_rounds: List[tuple] = dataclasses.field(default_factory=list)
+
+
+def _step1(target: Transformer, draft: Transformer, st: PromptState, run: RunParams, w_head,
+           dec: "Decider", b: int, L: int, roots, r_full, vlog, am, tc, dc, X: List[tuple],
+           rounds: List[tuple]) -> bool:
+    """Step-1 of Alg. 1's S2/S3 branch (Sec. 3.2.3) in the CDSL-k step, budget run.b.
+
+    Round 1: M_p's greedy token after pfx is the root c_1 and its d-token M_q lookahead is beam
+    1's draft, so its reward is r_1^full (data the step already has). Round i > 1: the next
+    token is M_p's argmax after pfx + X (round 2: verify row (1, 0)), its lookahead is d greedy
+    M_q tokens after pfx + X + token, and the reward is R(T + X + token + lh) with M_p's hidden
+    state at lh_d. The first round whose reward reaches r_t ends Step-1 with X emitted.
+
+    Appends (token, M_p cache through it, M_q cache through it, M_p logits after it) to X for
+    every round taken and (token + lh, reward) to ``rounds`` for rounds > 1. True on success."""
+    d = run.d
+    c1 = int(roots[0])
+    X.append((c1, tc[(b, 0)].truncated(L + 1), dc[(b, 0)].truncated(L + 1), vlog[0, 0]))
+    if dec.reward_ok(r_full[0], run.r_t, "step1", b):
+        return True
+    for i in range(1, run.b):
+        _, tcx, dcx, p_after = X[-1]
+        tok = int(am[0, 0]) if i == 1 else dec.argmax(p_after, "step1_tok", (b, i))
+        dce = dcx.fork()
+        lg, _ = draft.forward([(dce, [tok])])
+        lh = []
+        for j in range(d):
+            t = dec.argmax(lg[0][-1], "step1_x", (b, i, j))
+            lh.append(t)
+            if j + 1 < d:
+                lg, _ = draft.forward([(dce, [t])])
+        tce = tcx.fork()
+        vl2, vh2 = target.forward([(tce, [tok] + lh)])
+        span = [t for t, _, _, _ in X] + [tok] + lh
+        r = reward(st.keywords, st.T + span, vh2[0][d], w_head, run.composite_reward)
+        n_x = len(X) + 1
+        X.append((tok, tce.truncated(L + n_x), dce.truncated(L + n_x), vl2[0][0]))
+        rounds.append((np.asarray([tok] + lh, dtype=np.int64), r))
+        if dec.reward_ok(r, run.r_t, f"step1_{i + 1}", b):
+            return True
+    return False
 
 
 def cdsl_k_step(target: Transformer, draft: Transformer, states: List[PromptState],
@@ -355,16 +399,20 @@ def cdsl_k_step(target: Transformer, draft: Transformer, states: List[PromptStat
         # 6. beam
         bs = dec.first_max(r_full, "beam", b)
         # 7. state and emission
+        L = len(st.prompt) + len(st.T)
+        rounds: List[tuple] = []
+        X: List[int] = []
         if n[bs] >= nmin and dec.reward_ok(r_acc[bs], run.r_t, "s1", b):
             state = S1
             out = [int(roots[b][bs])] + x[b][bs, :n[bs]].tolist()
-        elif (n[bs] < nmin and run.b >= 1
-              and dec.reward_ok(r_full[0], run.r_t, "step1", b)):
-            # S2/S3, Step-1 with b = 1 (Alg. 1, Sec. 3.2.3): M_p's greedy token is c_1; its
-            # d-token M_q lookahead is beam 1's draft, scored R(T + c_1 + lh) = r_1^full
+        elif n[bs] < nmin and run.b >= 1 and _step1(target, draft, st, run, w_head, dec, b, L,
+                                                    roots[b], r_full, vlog, am, tc, dc, X,
+                                                    rounds):
+            # S2/S3, Step-1 (Alg. 1, Sec. 3.2.3): X = M_p's greedy tokens, the last of which
+            # had a lookahead reward >= r_t
             state = S2_S3_STEP1
             bs = 0
-            out = [int(roots[b][0])]
+            out = [t for t, _, _, _ in X]
         else:
             state = S2_S3 if n[bs] < nmin else S4
             out = [int(roots[b][bs])]
@@ -372,17 +420,23 @@ def cdsl_k_step(target: Transformer, draft: Transformer, states: List[PromptStat
         out = out[:n_emit]
 
         # commit: pfx <- pfx + O. The winner's caches hold exactly these positions.
-        L = len(st.prompt) + len(st.T)
-        st.tcache = tc[(b, bs)].truncated(L + n_emit)
-        st.p_root = vlog[bs, n_emit - 1]
-        st.h_root = vhid[bs, n_emit - 1]
-        # the winner's draft cache holds [c, x_1..x_{d-1}]; x_d (full accept) is run now
-        st.dcache = dc[(b, bs)].truncated(L + min(n_emit, d))
-        if n_emit == d + 1:
-            draft.forward([(st.dcache, [out[d]])])
+        if state == S2_S3_STEP1 and n_emit >= 2:
+            _, tcx, dcx, p_after = X[n_emit - 1]
+            st.tcache = tcx.truncated(L + n_emit)
+            st.p_root = p_after
+            st.h_root = None
+            st.dcache = dcx.truncated(L + n_emit)
+        else:
+            st.tcache = tc[(b, bs)].truncated(L + n_emit)
+            st.p_root = vlog[bs, n_emit - 1]
+            st.h_root = vhid[bs, n_emit - 1]
+            # the winner's draft cache holds [c, x_1..x_{d-1}]; x_d (full accept) is run now
+            st.dcache = dc[(b, bs)].truncated(L + min(n_emit, d))
+            if n_emit == d + 1:
+                draft.forward([(st.dcache, [out[d]])])
         st.T = st.T + out
         recs[b] = StepRecord(True, np.asarray(roots[b]), x[b], logq[b], vlog, am, logp, n,
-                             r_full, r_acc, head, bs, state, out)
+                             r_full, r_acc, head, bs, state, out, rounds)
     return recs
 
 

@@ -448,3 +448,113 @@ def test_step1_with_one_beam_changes_no_token():
         rb = cdsl_k_step(tgt, drf, b, run_params(k=1, d=3, r_t=0.4, b=1), w, step=step)[0]
         assert ra.emitted == rb.emitted
         assert (ra.state == rb.state) or (ra.state == S2_S3 and rb.state == oracle.S2_S3_STEP1)
+
+
+# ---------------------------------------------------------------- Step-1 with b = 2 (f2)
+
+def _fork_state(st):
+    import dataclasses
+    return dataclasses.replace(st, T=list(st.T), tcache=st.tcache.fork(), dcache=st.dcache.fork())
+
+
+def test_step1_second_round_emits_two_greedy_tokens():
+    """b = 2 with M_q = M_p, a_t above 1 (every step is S2/S3) and r_t = 1 on a single keyword
+    that M_p's greedy text reaches only at token d + 2: round 1 (c_1 + its lookahead, tokens
+    g_1..g_{d+1}) misses it, round 2 (g_1, g_2 + lookahead g_3..g_{d+2}) covers it, so the
+    step emits M_p's first two greedy tokens. With b = 1 the same step falls back to Step-2."""
+    d = 3
+    shp = shape(vocab=24)
+    tgt = model(shp, 17)
+    found = 0
+    for p0 in range(12):
+        prompt = [p0 % 24, (3 * p0 + 1) % 24, (5 * p0 + 2) % 24, 7]
+        g = greedy_chain(tgt, prompt, d + 2)
+        if g[d + 1] in g[:d + 1] or g[d + 1] in prompt:
+            continue
+        found += 1
+        kw = np.array([[g[d + 1]]])
+        for b, want_state, want_out in ((2, oracle.S2_S3_STEP1, g[:2]), (1, S2_S3, None)):
+            st = prefill(tgt, tgt, np.array([prompt]), kw)
+            run = run_params(k=3, d=d, a_t=1.5, r_t=1.0, composite_reward=False, b=b)
+            rec = cdsl_k_step(tgt, tgt, st, run, np.zeros(shp.d_model), step=0)[0]
+            assert rec.state == want_state
+            if b == 2:
+                assert rec.emitted == want_out and rec.beam == 0
+                (toks, r), = rec.step1_rounds
+                assert toks.tolist() == g[1:d + 2] and r == 1.0
+                # the committed caches continue M_p's greedy text
+                nxt = cdsl_k_step(tgt, tgt, st, run_params(k=3, d=d, a_t=1.5, r_t=-np.inf,
+                                                           composite_reward=False, b=1),
+                                  np.zeros(shp.d_model), step=1)[0]
+                assert nxt.emitted == [g[2]]
+            else:
+                assert len(rec.emitted) == 1 and rec.step1_rounds == []
+        if found >= 3:
+            break
+    assert found >= 3
+
+
+def test_step1_second_round_truncated_at_l_m():
+    """A Step-1 success in round 2 with one token left before l_m emits c_1 alone."""
+    d = 2
+    shp = shape(vocab=24)
+    tgt = model(shp, 23)
+    for p0 in range(12):
+        prompt = [p0, (7 * p0 + 3) % 24, 11]
+        g = greedy_chain(tgt, prompt, d + 2)
+        if g[d + 1] in g[:d + 1] or g[d + 1] in prompt:
+            continue
+        st = prefill(tgt, tgt, np.array([prompt]), np.array([[g[d + 1]]]))
+        run = run_params(k=2, d=d, a_t=1.5, r_t=1.0, composite_reward=False, b=2, max_new=1)
+        rec = cdsl_k_step(tgt, tgt, st, run, np.zeros(shp.d_model), step=0)[0]
+        assert rec.state == oracle.S2_S3_STEP1 and rec.emitted == [g[0]] and st[0].T == [g[0]]
+        return
+    pytest.fail("no prompt with a fresh keyword at greedy position d + 2")
+
+
+@pytest.mark.parametrize("r_t, same_as", [(0.0, 1), (np.inf, 0)])
+def test_step1_budget2_limits(r_t, same_as):
+    """r_t = 0: round 1 always succeeds, so b = 2 runs exactly like b = 1; r_t = inf: no round
+    succeeds, so b = 2 emits exactly what b = 0 does (Step-2)."""
+    shp = shape(vocab=24)
+    tgt, drf = model(shp, 51), model(shp, 52)
+    w = np.random.default_rng(53).standard_normal(shp.d_model)
+    prompts = np.array([[1, 2, 3, 4], [5, 6, 7, 8]])
+    kw = np.array([[1, 2, 3], [4, 5, 6]])
+    a, c = prefill(tgt, drf, prompts, kw), prefill(tgt, drf, prompts, kw)
+    for step in range(4):
+        ra = cdsl_k_step(tgt, drf, a, run_params(r_t=r_t, a_t=0.6, b=same_as), w, step=step)
+        rc = cdsl_k_step(tgt, drf, c, run_params(r_t=r_t, a_t=0.6, b=2), w, step=step)
+        for x, y in zip(ra, rc):
+            assert x.emitted == y.emitted and x.state == y.state and x.beam == y.beam
+    assert [s.T for s in a] == [s.T for s in c]
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2, 3])
+def test_step1_rounds_match_literal_algorithm1(seed):
+    """k = 1 and a step with no accepted draft (n = 0) in S2/S3: the batched step's Step-1 and
+    literal Algorithm 1's Step-1 (which starts after the accepted drafts, here none) take the
+    same greedy tokens, the same lookaheads and the same rewards, so with b = 2 they emit the
+    same tokens. The two share no Step-1 code."""
+    shp = shape(vocab=20)
+    dshp = shape(vocab=20, d=16, layers=1, heads=2, kv=1, ffn=20)
+    tgt, drf = model(shp, 60 + seed), model(dshp, 70 + seed)
+    w = np.random.default_rng(80 + seed).standard_normal(shp.d_model)
+    rng = np.random.default_rng(90 + seed)
+    compared = {1: 0, 2: 0, 0: 0}
+    for trial in range(16):
+        prompt = rng.integers(0, 20, size=5).tolist()
+        kw = rng.choice(20, size=3, replace=False).tolist()
+        r_t = float(rng.uniform(0.3, 0.7))
+        run = run_params(k=1, d=3, a_t=0.9, r_t=r_t, b=2, max_new=4)
+        lit = oracle.alg1_generate(tgt, drf, prompt, kw, run, w, max_steps=1)[1][0]
+        if lit["n"] != 0 or lit["state"] != S2_S3:
+            continue
+        st = prefill(tgt, drf, np.array([prompt]), np.array([kw]))
+        rec = cdsl_k_step(tgt, drf, st, run, w, step=0)[0]
+        if rec.state not in (S2_S3, oracle.S2_S3_STEP1):   # its own draft (after c_1) passed
+            continue
+        # literal Alg. 1 emits X after Step-1 success, else CDLH-appx's token (k = 1: c_1)
+        assert rec.emitted == lit["emitted"]
+        compared[0 if rec.state == S2_S3 else len(rec.emitted)] += 1
+    assert min(compared.values()) >= 1   # Step-2, round-1 and round-2 outcomes all compared
