@@ -40,7 +40,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--acceptance", choices=["hard", "speculative"], default="hard",
                     help="validation of the lookaheads by M_p (Sec. 3.2.2)")
-    ap.add_argument("--step1-budget", type=int, choices=[0, 1], default=0,
+    ap.add_argument("--step1-budget", type=int, choices=[0, 1, 2], default=0,
                     help="Alg. 1 S2/S3 Step-1 budget b (Sec. 3.2.3)")
     ap.add_argument("--decoder", choices=["cdsl", "cdlh", "cdlh-appx"], default="cdsl",
                     help="cdlh: the lookaheads come from M_p itself and no lookahead is ever "

@@ -14,8 +14,10 @@
  * a_b = n_b/d, the rewards, the chosen beam b* (largest r^full, first on ties) and the state:
  *   S1  (a_b* >= a_t and r^acc_b* >= r_t): emit c_b*, x_b*,1..n       (Sec. 3.2.3, S1)
  *   S2/S3 (a < a_t), S4 (a >= a_t, r < r_t): emit c_b* only, i.e. the one CDLH-appx token of
- *   Algorithm 1's fallback (Step-2); with a Step-1 budget b = 1 (cdsl_run_cfg.step1_budget),
- *   S2/S3 first emits M_p's greedy token c_1 if r^full_1 >= r_t (state 3).
+ *   Algorithm 1's fallback (Step-2); with a Step-1 budget b >= 1 (cdsl_run_cfg.step1_budget),
+ *   S2/S3 first tries M_p's greedy tokens: c_1 if r^full_1 >= r_t, and with b = 2 then
+ *   c_1, x' (x' = M_p's argmax after c_1) if the reward of x''s own lookahead reaches r_t
+ *   (state 3).
  *
  * Conventions
  *  - Every compute call is asynchronous on the stream given to cdsl_init (a cudaStream_t
@@ -99,10 +101,16 @@ typedef struct cdsl_run_cfg {
    * steps of the context (SplitMix64: Steele, Lea, Flood, OOPSLA 2014). */
   int32_t acceptance;
   uint32_t seed;
-  /* Step-1 budget b of Alg. 1's S2/S3 branch (Sec. 3.2.3), 0 or 1. With b = 1, a
-   * step in S2/S3 (a < a_t) first tries M_p's greedy token, the root c_1, whose draft
+  /* Step-1 budget b of Alg. 1's S2/S3 branch (Sec. 3.2.3), 0, 1 or 2. With b >= 1,
+   * a step in S2/S3 (a < a_t) first tries M_p's greedy token, the root c_1, whose draft
    * lookahead and reward r_1^full the step already has: if r_1^full >= r_t it emits c_1
-   * (state 3) instead of the CDLH-appx token c_{b*} of Step-2. */
+   * (state 3) instead of the CDLH-appx token c_{b*} of Step-2. With b = 2, when that fails,
+   * round 2 takes x' = argmax M_p(pfx + c_1) (verify row (b, 1, 0)), runs d greedy draft
+   * calls from pfx + c_1 + x' (lookahead lh) and one target pass over [x', c_1, lh] (for
+   * M_p(pfx + c_1 + x'), the reward head at lh_d and the K/V of c_1, x'), and emits c_1, x'
+   * (state 3) if R(T + c_1 + x' + lh) >= r_t. The round runs every step for every prompt
+   * (d extra draft calls and one extra target pass per step); only prompts whose round 1
+   * failed in S2/S3 use it. cdsl_get_step1 returns its tokens and rewards. */
   int32_t step1_budget;
 } cdsl_run_cfg;
 
@@ -155,13 +163,15 @@ CDSL_API int32_t cdsl_lookahead(cdsl_ctx* ctx, int32_t* d_roots, int32_t* d_draf
 CDSL_API int32_t cdsl_verify(cdsl_ctx* ctx, float* d_logp, int32_t* d_argmax, int32_t* d_n_accept,
                     float* d_logits);
 
-/* Acceptance decision and commit (Sec. 3.2.3, Algorithm 1 with b = 0 or 1): rewards
+/* Acceptance decision and commit (Sec. 3.2.3, Algorithm 1 with b = 0, 1 or 2): rewards
  * d_reward [B, k, 2] = (r^full, r^acc) per beam, d_beam [B] the beam whose tokens are
  * emitted (b*, or 0 for a Step-1 token), d_state [B] 1 (S1), 2 (S2/S3), 3 (S2/S3 resolved by
  * Step-1) or 4 (S4), d_emitted [B, d+1] the emitted tokens (-1 padded), d_n_emitted [B]
  * (0 for prompts that already hold l_m tokens). Emission is cut at l_m. Then the winner's KV
  * rows are committed to the prefix pages and the next beams are taken from the winner's
- * verify row. Requires a preceding cdsl_verify. */
+ * verify row (after a round-2 Step-1 emission: from M_p(pfx + c_1 + x')). With budget 2 the
+ * call also runs the Step-1 round (see cdsl_run_cfg.step1_budget). Requires a preceding
+ * cdsl_verify. */
 CDSL_API int32_t cdsl_select(cdsl_ctx* ctx, int32_t* d_beam, int32_t* d_state, int32_t* d_emitted,
                     int32_t* d_n_emitted, float* d_reward);
 
@@ -200,6 +210,12 @@ CDSL_API int32_t cdsl_get_profile(cdsl_ctx* ctx, int32_t impl, double* h_out);
  * [4 * i]; returns the number of records written (>= 0) or a negative status. Synchronizes
  * the stream. */
 CDSL_API int32_t cdsl_get_profile_launches(cdsl_ctx* ctx, double* h_out, int32_t h_capacity);
+
+/* Step-1 round 2 of the last cdsl_select / cdsl_step (budget 2; Alg. 1): d_need [B]
+ * 1 where round 1 failed in S2/S3 so that round 2 decided the step, d_tokens [B, d+1] the
+ * round's x' and lookahead lh_1..lh_d, d_reward [B] R(T + c_1 + x' + lh) (meaningful where
+ * d_need = 1). Any pointer may be NULL. CDSL_EINVAL with a smaller budget. */
+CDSL_API int32_t cdsl_get_step1(cdsl_ctx* ctx, int32_t* d_need, int32_t* d_tokens, float* d_reward);
 
 /* Synchronize the stream and return the device status word (a cdsl_status; CDSL_OK when no
  * device-side error was latched) in *h_device_status. Clears nothing. */

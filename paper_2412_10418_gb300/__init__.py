@@ -62,6 +62,7 @@ EXPORTS = {
     "cdsl_step": (_I, [_P, _P, _P, _P, _P, _P]),
     "cdsl_get_tokens": (_I, [_P, _P, _P]),
     "cdsl_get_counters": (_I, [_P, ctypes.POINTER(ctypes.c_int64)]),
+    "cdsl_get_step1": (_I, [_P, _P, _P, _P]),
     "cdsl_get_status": (_I, [_P, ctypes.POINTER(ctypes.c_int32)]),
     "cdsl_profile": (_I, [_P, _I]),
     "cdsl_get_profile": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double)]),
@@ -180,6 +181,10 @@ def cdsl_get_counters(ctx) -> List[int]:
     return list(out)
 
 
+def cdsl_get_step1(ctx, need=None, tokens=None, reward=None):
+    _check(lib().cdsl_get_step1(ctx, _ptr(need), _ptr(tokens), _ptr(reward)), ctx)
+
+
 def cdsl_get_status(ctx) -> int:
     v = ctypes.c_int32(0)
     _check(lib().cdsl_get_status(ctx, ctypes.byref(v)), ctx)
@@ -290,6 +295,17 @@ class Engine:
         cdsl_get_tokens(self.ctx, t, n)
         self.stream.synchronize()
         return t, n
+
+    def step1(self):
+        """Step-1 round 2 of the last select / step (budget 2): need [B], tokens [B, d+1]
+        (x', lh_1..lh_d), reward [B]."""
+        t = self.torch
+        need = t.zeros(self.B, dtype=t.int32, device=self.ws.device)
+        tok = t.zeros((self.B, self.d + 1), dtype=t.int32, device=self.ws.device)
+        rew = t.zeros(self.B, dtype=t.float32, device=self.ws.device)
+        cdsl_get_step1(self.ctx, need, tok, rew)
+        self.stream.synchronize()
+        return need, tok, rew
 
     def counters(self):
         return cdsl_get_counters(self.ctx)

@@ -58,7 +58,7 @@ struct cdsl_ctx {
   const float* head_w = nullptr;
   int dtype = 0;
   int B = 0, k = 0, d = 0, nk = 0, lcap = 0, lrope = 0, max_pages = 0, page_shift = 0;
-  int R_v = 0, R_d = 0, R_p = 0, R_max = 0, R_pad = 0, V = 0;
+  int R_v = 0, R_d = 0, R_p = 0, R_s1 = 0, R_max = 0, R_pad = 0, V = 0;
   int d_max = 0, act_cols = 0, q_cols = 0;
   size_t act_plane = 0;  // elements between hi and lo planes of X1 / X2 (bf16 models)
   // buffers
@@ -155,8 +155,7 @@ int check_run(const cdsl_run_cfg* r, int vocab, std::string* why) {
   if (r->max_chunk < 0) return bad("max_chunk must be >= 0");
   if (r->acceptance != 0 && r->acceptance != 1)
     return bad("acceptance must be 0 (hard rejection) or 1 (speculative sampling)");
-  if (r->step1_budget != 0 && r->step1_budget != 1)
-    return bad("step1_budget must be 0 or 1");
+  if (r->step1_budget < 0 || r->step1_budget > 2) return bad("step1_budget must be 0, 1 or 2");
   return CDSL_OK;
 }
 
@@ -164,10 +163,25 @@ int group_size(const cdsl_model_cfg& m) { return m.n_heads / m.n_kv_heads; }
 int prefix_chunks(const cdsl_run_cfg& r) {
   return (r.max_prompt + r.max_new + attn_chunk() - 1) / attn_chunk();
 }
-// Most tail-key chunks of any pass: the verify rows of the target, the draft rollout rows.
+// Tail-key chunks of the Step-1 round's passes (budget 2): the target's d+2 rows per prompt
+// and the draft's (at most 2 rows, d+1 tail slots).
+int s1_tail_chunks_t(const cdsl_model_cfg& t, const cdsl_run_cfg& r) {
+  return attn_tail_chunks(r.d + 2, group_size(t), r.d + 2, r.d + 2);
+}
+int s1_tail_chunks_d(const cdsl_model_cfg& dr, const cdsl_run_cfg& r, int j) {
+  const int rows = j == 1 ? 2 : 1;
+  return attn_tail_chunks(rows, group_size(dr), rows, j + 1);
+}
+// Most tail-key chunks of any pass: the verify rows of the target, the draft rollout rows
+// (and the Step-1 round's passes).
 int tail_chunks_max(const cdsl_model_cfg& t, const cdsl_model_cfg& dr, const cdsl_run_cfg& r) {
-  return std::max(attn_tail_chunks(r.k * (r.d + 1), group_size(t), r.d + 1, r.d + 1),
-                  attn_tail_chunks(r.k + 1, group_size(dr), 1, r.d));
+  int m = std::max(attn_tail_chunks(r.k * (r.d + 1), group_size(t), r.d + 1, r.d + 1),
+                   attn_tail_chunks(r.k + 1, group_size(dr), 1, r.d));
+  if (r.step1_budget >= 2) {
+    m = std::max(m, s1_tail_chunks_t(t, r));
+    for (int j = 1; j <= r.d; ++j) m = std::max(m, s1_tail_chunks_d(dr, r, j));
+  }
+  return m;
 }
 
 // Sizes derived from the configurations (shared by cdsl_workspace_size and cdsl_init).
@@ -184,11 +198,13 @@ void derive_dims(cdsl_ctx* c) {
   c->max_pages = (c->lcap + ps - 1) / ps;
   c->R_v = c->B * c->k * (c->d + 1);
   c->R_d = c->B * c->k + c->B;
+  // Step-1 round 2: the target pass holds d+2 rows per prompt (draft calls fit in R_d)
+  c->R_s1 = r.step1_budget >= 2 ? c->B * (c->d + 2) : 0;
   // default 64 prefill rows: the projections then stay on the fused hi/lo MMA with two blocks
   // per SM (measured: 54 ms for the 512-token 7B prefill, against 96 ms at 256 rows)
   const int chunk = r.max_chunk ? r.max_chunk : 64;
   c->R_p = std::min(chunk, c->B * r.max_prompt);
-  c->R_max = std::max(c->R_v, std::max(c->R_d, c->R_p));
+  c->R_max = std::max(std::max(c->R_v, c->R_s1), std::max(c->R_d, c->R_p));
   c->R_pad = (c->R_max + 31) / 32 * 32;
   c->d_max = std::max(c->tcfg.d_model, c->dcfg.d_model);
   c->q_cols = std::max(c->tcfg.n_heads * c->tcfg.head_dim, c->dcfg.n_heads * c->dcfg.head_dim);
@@ -211,17 +227,21 @@ KvStore make_kv(const cdsl_model_cfg& m, cdsl_ctx* c, int slots) {
 size_t carve(cdsl_ctx* c, void* base) {
   Carver cv(base);
   const int B = c->B, k = c->k, d = c->d;
-  auto model_kv = [&](ModelW& m, const cdsl_model_cfg& cfg, int slots) {
+  auto model_kv = [&](ModelW& m, const cdsl_model_cfg& cfg, int spb, int extra) {
+    const int slots = B * k * spb + extra;
     m.kv = make_kv(cfg, c, slots);
     const size_t per_page = (size_t)2 * cfg.n_kv_heads * ((size_t)1 << c->page_shift) * cfg.head_dim;
     m.kv.pool = cv.take<float>((size_t)cfg.n_layers * m.kv.n_pages * per_page);
     m.kv.tail = cv.take<float>((size_t)cfg.n_layers * 2 * slots * cfg.n_kv_heads * cfg.head_dim);
     m.kv.page_table = cv.take<int32_t>((size_t)B * c->max_pages);
     m.rope = cv.take<float2>((size_t)c->lrope * (cfg.head_dim / 2));
-    m.spb = slots / (B * k);
+    m.spb = spb;
   };
-  model_kv(c->tgt, c->tcfg, B * k * (d + 1));
-  model_kv(c->dft, c->dcfg, B * k * d);
+  // per beam: target d+1 verify rows, draft d rollout rows; the Step-1 round (budget 2) adds
+  // d+2 target and d+1 draft slots per prompt after them
+  const bool s1 = c->run.step1_budget >= 2;
+  model_kv(c->tgt, c->tcfg, d + 1, s1 ? B * (d + 2) : 0);
+  model_kv(c->dft, c->dcfg, d, s1 ? B * (d + 1) : 0);
   c->h = cv.take<float>((size_t)c->R_pad * c->d_max);
   // GEMM inputs: one fp32 plane, or hi/lo bf16 planes (4 bytes per element either way)
   c->act_plane = (size_t)c->R_pad * c->act_cols;
@@ -236,7 +256,7 @@ size_t carve(cdsl_ctx* c, void* base) {
   const int lm_rows = std::max(c->R_v, std::max(B * k, B));
   c->logits = cv.take<float>((size_t)lm_rows * c->V);
   c->rows_d = cv.take<RowDesc>(c->R_d);
-  c->rows_v = cv.take<RowDesc>(c->R_v);
+  c->rows_v = cv.take<RowDesc>(std::max(c->R_v, c->R_s1));
   c->rows_p = cv.take<RowDesc>(c->R_p);
   c->lm_gather = cv.take<int32_t>(c->R_p);
   c->lm_dst = cv.take<int32_t>(c->R_p);
@@ -277,6 +297,8 @@ size_t carve(cdsl_ctx* c, void* base) {
   s.acceptance = c->run.acceptance;
   s.seed = c->run.seed;
   s.step1 = c->run.step1_budget;
+  s.s1_tbase = B * k * (d + 1);
+  s.s1_dbase = B * k * d;
   s.n_min = d + 1;
   for (int n = 0; n <= d; ++n)
     if ((float)n / (float)d >= c->run.a_t) { s.n_min = n; break; }
@@ -302,6 +324,12 @@ size_t carve(cdsl_ctx* c, void* base) {
   s.next_page = cv.take<int32_t>(2);
   s.status = cv.take<int32_t>(1);
   s.counters = cv.take<long long>(8);
+  s.s1_need = cv.take<int32_t>(B);
+  s.s1_tok = cv.take<int32_t>((size_t)B * (d + 1));
+  s.s1_logq = cv.take<float>((size_t)B * (d + 1));
+  s.s1_reward = cv.take<float>(B);
+  s.s1_topk = cv.take<int32_t>((size_t)B * k);
+  s.s1_used = cv.take<int32_t>(B);
   return (cv.off + 255) & ~size_t(255);
 }
 
@@ -537,9 +565,43 @@ void do_verify(cdsl_ctx* c) {
   timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
 }
 
-void do_select(cdsl_ctx* c) {
+// Step-1 round 2 (Alg. 1 S2/S3, budget b = 2) for every prompt: d draft calls from
+// pfx + c_1 + x' and one target pass over [x', c_1, lh_1..lh_d]; k_select_s1 then keeps the
+// Step-2 emission or replaces it with c_1, x'. The round's work is the same every step (the
+// graph is static); only prompts whose round 1 failed in S2/S3 use its result.
+void do_step1_round(cdsl_ctx* c) {
+  const int B = c->B, d = c->d;
+  for (int j = 1; j <= d; ++j) {
+    timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_s1_draft(c->st, j, c->rows_d, c->stream); });
+    AttnPass ap;
+    ap.rows_per_prompt = j == 1 ? 2 : 1;
+    ap.n_tchunks = s1_tail_chunks_d(c->dcfg, c->run, j);
+    forward(c, c->dft, c->rows_d, ap.rows_per_prompt * B, B, nullptr, c->logits, false, ap);
+    RowStatsArgs a{};
+    a.logits = c->logits; a.R = B; a.V = c->V; a.k = c->k;
+    a.x_out = c->st.s1_tok; a.logq_out = c->st.s1_logq; a.out_stride = d + 1; a.out_off = j;
+    a.status = c->st.status;
+    timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
+  }
+  timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_s1_verify(c->st, c->rows_v, c->stream); });
+  AttnPass ap;
+  ap.rows_per_prompt = d + 2;
+  ap.n_tchunks = s1_tail_chunks_t(c->tcfg, c->run);
+  forward(c, c->tgt, c->rows_v, c->R_s1, B, nullptr, c->logits, c->run.reward_head != 0, ap);
+  RowStatsArgs a{};
+  a.logits = c->logits; a.R = B; a.V = c->V; a.k = c->k;
+  a.topk = c->st.s1_topk; a.status = c->st.status;
+  timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
   timed(c, K_STEPLOGIC, 0, 0, [&] {
-    launch_select(c->st, c->tgt.kv, c->dft.kv, 1, c->stream);
+    launch_select_s1(c->st, c->tgt.kv, c->dft.kv, c->ss_a, c->ss_hw, c->tcfg.d_model, c->R_pad,
+                     c->tcfg.norm_eps, c->stream);
+  });
+}
+
+void do_select(cdsl_ctx* c) {
+  timed(c, K_STEPLOGIC, 0, 0, [&] { launch_select(c->st, c->tgt.kv, c->dft.kv, 1, c->stream); });
+  if (c->run.step1_budget >= 2) do_step1_round(c);
+  timed(c, K_STEPLOGIC, 0, 0, [&] {
     launch_commit_kv(c->st, c->tgt.kv, c->tgt.spb, 0, c->stream);
     launch_commit_kv(c->st, c->dft.kv, c->dft.spb, 1, c->stream);
     launch_advance(c->st, c->stream);
@@ -913,6 +975,16 @@ int32_t cdsl_get_profile_launches(cdsl_ctx* c, double* h_out, int32_t h_capacity
     ++n;
   }
   return n;
+}
+
+int32_t cdsl_get_step1(cdsl_ctx* c, int32_t* d_need, int32_t* d_tokens, float* d_reward) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (c->run.step1_budget < 2) return fail(c, CDSL_EINVAL, "cdsl_get_step1 needs step1_budget 2");
+  const size_t B = c->B;
+  copy_out(c, d_need, c->st.s1_need, B * 4);
+  copy_out(c, d_tokens, c->st.s1_tok, B * (c->d + 1) * 4);
+  copy_out(c, d_reward, c->st.s1_reward, B * 4);
+  return cuda_check(c, "cdsl_get_step1");
 }
 
 int32_t cdsl_get_status(cdsl_ctx* c, int32_t* h_device_status) {

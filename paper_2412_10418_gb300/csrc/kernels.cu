@@ -275,6 +275,76 @@ __global__ void k_plan_verify(StepState st, RowDesc* rows) {
   rows[r] = rd;
 }
 
+// Step-1 round 2, draft call j (1..d), in the round's own tail region of d+1 slots per prompt
+// (slot 0 c_1, slot 1 x', slot j lh_j-1): rows [0, B) carry x' at L + 1 (j = 1, which also
+// records x' = argmax M_p(pfx + c_1), verify row (b, 1, 0)) or lh_j-1 at L + j; rows [B, 2B)
+// of call 1 carry c_1 at L.
+__global__ void k_plan_s1_draft(StepState st, int j, RowDesc* rows) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int B = st.B, dp1 = st.d + 1;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= (j == 1 ? 2 * B : B)) return;
+  const int b = r % B;
+  const int L = st.len[b], base = st.s1_dbase + b * dp1;
+  RowDesc rd;
+  rd.b = b;
+  rd.n_prefix = L;
+  rd.tail_base = base;
+  if (r >= B) {
+    rd.pos = L;
+    rd.token = st.roots[b * st.k];
+    rd.n_tail = 1;
+    rd.kv_dst = base;
+    rd.out_idx = -1;
+  } else if (j == 1) {
+    const int xp = st.v_amax[b * st.k * dp1];
+    st.s1_tok[b * dp1] = xp;
+    rd.pos = L + 1;
+    rd.token = xp;
+    rd.n_tail = 2;
+    rd.kv_dst = base + 1;
+    rd.out_idx = b;
+  } else {
+    rd.pos = L + j;
+    rd.token = st.s1_tok[b * dp1 + j - 1];
+    rd.n_tail = j + 1;
+    rd.kv_dst = base + j;
+    rd.out_idx = b;
+  }
+  rows[r] = rd;
+}
+
+// Step-1 round 2, the target pass, in its tail region of d+2 slots per prompt (c_1, x',
+// lh_1..lh_d): rows [0, B) x' at L + 1 (the LM rows: M_p(pfx + c_1 + x')), [B, 2B) c_1 at L,
+// then lh_j at L + 1 + j, prompt-major (the reward head reads lh_d's row).
+__global__ void k_plan_s1_verify(StepState st, RowDesc* rows) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int B = st.B, d = st.d, dp1 = d + 1;
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= B * (d + 2)) return;
+  int b, slot;
+  if (r < B) {
+    b = r; slot = 1;
+  } else if (r < 2 * B) {
+    b = r - B; slot = 0;
+  } else {
+    b = (r - 2 * B) / d; slot = 2 + (r - 2 * B) % d;
+  }
+  const int L = st.len[b], base = st.s1_tbase + b * (d + 2);
+  RowDesc rd;
+  rd.b = b;
+  rd.pos = L + slot;
+  rd.token = slot == 0 ? st.roots[b * st.k] : st.s1_tok[b * dp1 + slot - 1];
+  rd.n_prefix = L;
+  rd.tail_base = base;
+  rd.n_tail = slot + 1;
+  rd.kv_dst = base + slot;
+  rd.out_idx = r < B ? b : -1;
+  rows[r] = rd;
+}
+
 // ------------------------------------------------------------------------------ decision
 __device__ void alloc_pages(const KvStore& kv, int b, int from, int to, int32_t* next_page,
                             int32_t* status) {
@@ -314,7 +384,10 @@ __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
       st.n_acc[b * k + lane] = 0;
     }
     if (lane < dp1) st.emitted[b * dp1 + lane] = -1;
-    if (lane == 0) { st.beam[b] = -1; st.state[b] = 0; st.n_emit[b] = 0; }
+    if (lane == 0) {
+      st.beam[b] = -1; st.state[b] = 0; st.n_emit[b] = 0;
+      st.s1_need[b] = 0; st.s1_used[b] = 0;
+    }
     return;
   }
   float rf = -INFINITY, ra = -INFINITY;
@@ -382,6 +455,9 @@ __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
     st.beam[b] = win;
     st.state[b] = s1 ? 1 : (step1 ? 3 : (nb < st.n_min ? 2 : 4));
     st.n_emit[b] = cnt;
+    // budget 2: round 1 failed in S2/S3, round 2 may still replace this Step-2 emission
+    st.s1_need[b] = (!s1 && nb < st.n_min && st.step1 >= 2 && !(rf1 >= st.r_t)) ? 1 : 0;
+    st.s1_used[b] = 0;
     if (!commit) return;
     const int L = st.len[b];
     alloc_pages(tkv, b, L, L + cnt, st.next_page + 0, st.status);
@@ -389,22 +465,71 @@ __global__ void k_select(StepState st, KvStore tkv, KvStore dkv, int commit) {
   }
 }
 
-// Copy the winner's tail K/V rows 0..cnt-1 to prefix positions L..L+cnt-1.
+// Step-1 round 2 (Alg. 1 S2/S3, Sec. 3.2.3, budget b = 2): X = [c_1, x'] with the lookahead
+// lh of x'; R(T + X + lh) from the keyword bits and M_p's hidden state at lh_d (the same
+// arithmetic as the verify rows' head). One warp per prompt.
+__global__ void k_select_s1(StepState st, KvStore tkv, KvStore dkv, const float* ss,
+                            const float* hw, int norm_D, int ld_ss, float eps) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int b = blockIdx.x, lane = threadIdx.x;
+  const int d = st.d, dp1 = d + 1;
+  if (!st.s1_need[b]) return;
+  const int c1 = st.roots[b * st.k];
+  uint32_t bits = 0;
+  if (lane < st.nk) {
+    const int kwq = st.kw[b * st.nk + lane];
+    bool hit = c1 == kwq;
+    for (int j = 0; j < dp1; ++j) hit |= st.s1_tok[b * dp1 + j] == kwq;
+    if (hit) bits = 1u << lane;
+  }
+  for (int o = 16; o > 0; o >>= 1) bits |= __shfl_xor_sync(0xffffffffu, bits, o);
+  const float cov = (float)__popc(st.cov[b] | bits) / (float)st.nk;
+  float r = cov;
+  if (st.reward_head) {
+    const int row = 2 * st.B + b * d + d - 1;   // lh_d
+    float h = 0.f;
+    for (int c = lane; c < (norm_D >> 5); c += 32) h += hw[(size_t)c * ld_ss + row];
+    h = warp_sum(h);
+    const float rs = row_scale(ss, norm_D >> 5, ld_ss, row, norm_D, eps);
+    r = 0.5f * cov + 0.5f * (1.0f / (1.0f + expf(-h * rs)));
+  }
+  if (lane == 0) st.s1_reward[b] = r;
+  if (!(r >= st.r_t)) return;   // Step-2 (the c_b* emission of k_select) stands
+  const int cnt = min(2, st.max_new - st.gen[b]);
+  if (lane < dp1)
+    st.emitted[b * dp1 + lane] = lane == 0 ? c1 : ((lane == 1 && cnt == 2) ? st.s1_tok[b * dp1] : -1);
+  if (lane == 0) {
+    st.beam[b] = 0;
+    st.state[b] = 3;
+    st.n_emit[b] = cnt;
+    st.s1_used[b] = cnt == 2 ? 1 : 0;   // one token left: c_1 from beam 1's tails
+    const int L = st.len[b];
+    alloc_pages(tkv, b, L, L + cnt, st.next_page + 0, st.status);
+    alloc_pages(dkv, b, L, L + cnt, st.next_page + 1, st.status);
+  }
+}
+
+// Copy the winner's tail K/V rows 0..cnt-1 to prefix positions L..L+cnt-1 (after a Step-1
+// round-2 emission: rows 0, 1 of the round's tail region).
 __global__ void k_commit_kv(StepState st, KvStore kv, int spb, int is_draft) {
   pdl_wait();
   pdl_launch_dependents();
   const int b = blockIdx.x, layer = blockIdx.y, kvsel = blockIdx.z;
   int cnt = st.n_emit[b];
-  if (is_draft) cnt = min(cnt, st.d);
+  const bool s1 = st.s1_used[b] != 0;
+  if (is_draft && !s1) cnt = min(cnt, st.d);
   if (cnt <= 0) return;
   const int bs = st.beam[b], L = st.len[b];
+  const int src0 = !s1 ? (b * st.k + bs) * spb
+                       : (is_draft ? st.s1_dbase + b * (st.d + 1) : st.s1_tbase + b * (st.d + 2));
   const int per_row = kv.kvh * kv.hd;
   for (int e = threadIdx.x; e < cnt * per_row; e += blockDim.x) {
     const int j = e / per_row, rest = e % per_row, head = rest / kv.hd, c = rest % kv.hd;
     const int pos = L + j;
     const int page = kv.page_table[b * kv.max_pages + (pos >> kv.page_shift)];
     if (page < 0) continue;
-    const float* src = kv.tail + kv_tail_offset(kv, layer, kvsel, (b * st.k + bs) * spb + j, head);
+    const float* src = kv.tail + kv_tail_offset(kv, layer, kvsel, src0 + j, head);
     float* dst = kv.pool + kv_prefix_offset(kv, layer, page, kvsel, head, pos & ((1 << kv.page_shift) - 1));
     dst[c] = src[c];
   }
@@ -417,9 +542,10 @@ __global__ void k_advance(StepState st) {
   const int b = blockIdx.x, lane = threadIdx.x;
   const int k = st.k, d = st.d, dp1 = d + 1;
   if (b == 0 && lane == 0) {
-    st.counters[0] += 1;       // steps
-    st.counters[1] += d;       // draft forward passes
-    st.counters[2] += 1;       // target forward passes
+    const int rounds = st.step1 >= 2 ? 2 : 1;   // the Step-1 round runs every step
+    st.counters[0] += 1;                        // steps
+    st.counters[1] += d * rounds;               // draft forward passes
+    st.counters[2] += rounds;                   // target forward passes
   }
   const int cnt = st.n_emit[b];
   if (cnt <= 0) return;
@@ -432,13 +558,15 @@ __global__ void k_advance(StepState st) {
       if (st.emitted[b * dp1 + t] == kwq) bits = 1u << lane;
   }
   for (int o = 16; o > 0; o >>= 1) bits |= __shfl_xor_sync(0xffffffffu, bits, o);
+  const bool s1 = st.s1_used[b] != 0;   // next roots: top-k of M_p(pfx + c_1 + x')
   const int root_row = (b * k + bs) * dp1 + cnt - 1;
-  if (lane < k) st.roots[b * k + lane] = st.v_topk[root_row * k + lane];
+  if (lane < k)
+    st.roots[b * k + lane] = s1 ? st.s1_topk[b * k + lane] : st.v_topk[root_row * k + lane];
   if (lane == 0) {
     st.cov[b] |= bits;
     st.len[b] = L + cnt;
     st.gen[b] += cnt;
-    st.pend[b] = (cnt == dp1) ? 1 : 0;
+    st.pend[b] = (!s1 && cnt == dp1) ? 1 : 0;
     atomicAdd((unsigned long long*)&st.counters[3], (unsigned long long)cnt);
     if (st.state[b] == 1) atomicAdd((unsigned long long*)&st.counters[4], 1ull);
     atomicAdd((unsigned long long*)&st.counters[5], 1ull);
@@ -495,6 +623,22 @@ void launch_plan_draft(const StepState& st, int j, int spb, RowDesc* rows, cudaS
 void launch_plan_verify(const StepState& st, RowDesc* rows, cudaStream_t s) {
   const int n = st.B * st.k * (st.d + 1);
   launch_pdl(k_plan_verify, dim3((n + 127) / 128), dim3(128), 0, s, st, rows);
+}
+
+void launch_plan_s1_draft(const StepState& st, int j, RowDesc* rows, cudaStream_t s) {
+  const int n = j == 1 ? 2 * st.B : st.B;
+  launch_pdl(k_plan_s1_draft, dim3((n + 127) / 128), dim3(128), 0, s, st, j, rows);
+}
+
+void launch_plan_s1_verify(const StepState& st, RowDesc* rows, cudaStream_t s) {
+  const int n = st.B * (st.d + 2);
+  launch_pdl(k_plan_s1_verify, dim3((n + 127) / 128), dim3(128), 0, s, st, rows);
+}
+
+void launch_select_s1(const StepState& st, KvStore tkv, KvStore dkv, const float* ss,
+                      const float* hw, int norm_D, int ld_ss, float norm_eps, cudaStream_t s) {
+  launch_pdl(k_select_s1, dim3(st.B), dim3(32), 0, s, st, tkv, dkv, ss, hw, norm_D, ld_ss,
+             norm_eps);
 }
 
 void launch_select(const StepState& st, KvStore tkv, KvStore dkv, int commit, cudaStream_t s) {

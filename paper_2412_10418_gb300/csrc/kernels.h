@@ -16,7 +16,9 @@ struct StepState {
   float r_t;
   int32_t acceptance;  // 0 hard rejection, 1 speculative sampling
   uint32_t seed;       // SplitMix64 seed of the speculative-sampling draws
-  int32_t step1;       // Step-1 budget b (0 or 1)
+  int32_t step1;       // Step-1 budget b (0, 1 or 2)
+  int32_t s1_dbase;    // Step-1 round 2: first draft tail slot of its region (d+1 per prompt)
+  int32_t s1_tbase;    //   and first target tail slot (d+2 per prompt)
   int32_t* len;        // [B] committed prefix length L (target; draft up to the pending row)
   int32_t* pend;       // [B] 1: the draft still lacks the KV of token L-1
   int32_t* gen;        // [B] tokens generated (len(T))
@@ -39,6 +41,13 @@ struct StepState {
   int32_t* next_page;  // [2] bump allocators (target, draft)
   int32_t* status;     // device status word
   long long* counters; // [8]
+  // Step-1 round 2 (budget b = 2): x' = argmax M_p(pfx + c_1), its d-token M_q lookahead
+  int32_t* s1_need;    // [B] 1: round 1 failed in S2/S3 and round 2 decides the step
+  int32_t* s1_tok;     // [B, d+1] x', lh_1..lh_d
+  float* s1_logq;      // [B, d+1] log q of lh_1..lh_d (index 1..d)
+  float* s1_reward;    // [B] R(T + c_1 + x' + lh)
+  int32_t* s1_topk;    // [B, k] top-k of M_p(pfx + c_1 + x')
+  int32_t* s1_used;    // [B] 1: c_1, x' were emitted (K/V from the round's tails)
 };
 
 // elementwise / row kernels (T = float or __nv_bfloat16, the model dtype)
@@ -130,8 +139,16 @@ void set_thread_error(const char* msg);
 void launch_plan_draft(const StepState& st, int j, int tail_slots_per_beam, RowDesc* rows,
                        cudaStream_t s);
 void launch_plan_verify(const StepState& st, RowDesc* rows, cudaStream_t s);
+// Step-1 round 2: draft call j (1..d) over [x' (+ c_1 when j = 1)] or lh_j-1, and the target
+// pass over [x', c_1, lh_1..lh_d] of every prompt
+void launch_plan_s1_draft(const StepState& st, int j, RowDesc* rows, cudaStream_t s);
+void launch_plan_s1_verify(const StepState& st, RowDesc* rows, cudaStream_t s);
 // commit = 0: decide only (n_b, rewards, b*, state, emission); 1: also allocate KV pages
 void launch_select(const StepState& st, KvStore tkv, KvStore dkv, int commit, cudaStream_t s);
+// Step-1 round 2's decision: R(T + c_1 + x' + lh) >= r_t emits c_1, x' (state 3). ss / hw:
+// the target pass's final-norm and reward-head partial sums (ld_ss rows apart).
+void launch_select_s1(const StepState& st, KvStore tkv, KvStore dkv, const float* ss,
+                      const float* hw, int norm_D, int ld_ss, float norm_eps, cudaStream_t s);
 void launch_commit_kv(const StepState& st, KvStore kv, int slots_per_beam, int is_draft,
                       cudaStream_t s);
 void launch_advance(const StepState& st, cudaStream_t s);

@@ -92,6 +92,10 @@ def gpu_step_outputs(eng, with_logits=True):
            ("roots", "draft_tok", "logq", "logp", "argmax", "n_accept", "beam", "state",
             "emitted", "n_emitted", "reward")}
     out["logits"] = lg.cpu().numpy() if with_logits else None
+    if eng.run.step1_budget >= 2:
+        need, tok, rew = eng.step1()
+        out["s1_need"], out["s1_tok"], out["s1_reward"] = (need.cpu().numpy(), tok.cpu().numpy(),
+                                                           rew.cpu().numpy())
     return out
 
 
@@ -120,6 +124,12 @@ def compare_step(g, recs, tol, tol_r, report):
         ne = int(g["n_emitted"][b])
         assert g["emitted"][b][:ne].tolist() == rec.emitted, f"{where}: emitted"
         assert np.all(g["emitted"][b][ne:] == -1)
+        if "s1_need" in g:   # Step-1 round 2 ran exactly where round 1 failed in S2/S3
+            assert bool(g["s1_need"][b]) == bool(rec.step1_rounds), f"{where}: step-1 round"
+            if rec.step1_rounds:
+                toks, r2 = rec.step1_rounds[0]
+                assert g["s1_tok"][b].tolist() == toks.tolist(), f"{where}: step-1 tokens"
+                worst["reward"] = max(worst["reward"], abs(float(g["s1_reward"][b]) - r2))
     for key, lim in (("logits", tol), ("logq", tol), ("logp", tol), ("reward", tol_r)):
         assert worst[key] <= lim, f"{key}: max |diff| {worst[key]:.3g} > {lim}"
         report.setdefault(key, 0.0)
@@ -130,9 +140,16 @@ def compare_step(g, recs, tol, tol_r, report):
 def decider_from(g, tol, tol_r):
     # a Step-1 token (state 3) reports beam 0, not b*: no beam choice to adopt there
     beam = np.where(g["state"] == oracle.S2_S3_STEP1, -1, g["beam"])
+    step1 = g["state"] == oracle.S2_S3_STEP1
     other = {"roots": g["roots"], "x": g["draft_tok"], "argmax": g["argmax"], "beam": beam,
-             "s1": g["state"] == oracle.S1, "step1": g["state"] == oracle.S2_S3_STEP1,
-             "spec": g["n_accept"]}
+             "s1": g["state"] == oracle.S1, "step1": step1, "spec": g["n_accept"]}
+    if "s1_need" in g:   # budget 2: round 1 decided where round 2 did not run
+        need = g["s1_need"].astype(bool)
+        other["step1"] = step1 & ~need
+        other["step1_2"] = step1 & need
+        x2 = np.zeros((g["s1_tok"].shape[0], 2, g["s1_tok"].shape[1] - 1), np.int64)
+        x2[:, 1, :] = g["s1_tok"][:, 1:]
+        other["step1_x"] = x2
     return oracle.Decider(other=other, tol=tol, tol_r=tol_r)
 
 
@@ -158,10 +175,14 @@ def run_parity(s: Setup, steps: int, tol: float, tol_r: float, eng=None, page_si
         compare_step(g, recs, tol, tol_r, report)
         report["accepted"] = report.get("accepted", 0) + int(
             sum(g["n_accept"][b].sum() for b, r in enumerate(recs) if r.active))
-        for r in recs:
+        for b, r in enumerate(recs):
             if r.active:
                 key = f"state{r.state}"
                 report[key] = report.get(key, 0) + 1
+                if r.step1_rounds:
+                    report["round2"] = report.get("round2", 0) + 1
+                    if r.state == oracle.S2_S3_STEP1:
+                        report["round2_ok"] = report.get("round2_ok", 0) + 1
         adopted += dec.adopted
         n_steps += 1
     assert eng.status() == 0

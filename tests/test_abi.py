@@ -81,7 +81,8 @@ def test_bad_model_config(cdsl, field, value, msg):
 
 
 @pytest.mark.parametrize("field,value", [("k", 0), ("k", 17), ("d", 0), ("n_keywords", 33),
-                                         ("page_size", 48), ("batch", 0)])
+                                         ("page_size", 48), ("batch", 0), ("acceptance", 2),
+                                         ("step1_budget", 3), ("step1_budget", -1)])
 def test_bad_run_config(cdsl, field, value):
     t, d, r = cfgs(cdsl)
     setattr(r, field, value)

@@ -237,6 +237,75 @@ def test_tiny_step1_mixed_states():
     print("step-1 states:", {k: v for k, v in rep.items() if k.startswith("state")})
 
 
+def test_tiny_step1_second_round_follows_greedy_text():
+    """Step-1 budget b = 2, one beam (k = 1: Step-2 emits c_1, M_p's greedy token), M_q = M_p,
+    a_t above 1 (every step S2/S3), r_t = 1 over keywords g_1, g_2 and g_p (M_p's greedy
+    tokens, p = d + 5): round 2, taking g_t+1, g_t+2 with lookahead g_t+3..g_t+d+2, first
+    covers g_p at t = 3: that step emits two tokens, after three single-token steps; then
+    round 1 succeeds every step. The whole generation is M_p's greedy text, GPU and oracle
+    step by step (with k = 1 the round's d+2 target rows outnumber the verify rows)."""
+    wl = synth.scaled(synth.TINY, k=1, a_t=1.5, r_t=1.0, max_new=12)
+    t_host = synth.model_weights(wl, "target", device="host")
+    tgt = oracle.Transformer(wl.target, t_host)
+    p = synth.prompts(wl)[0].tolist()
+    g = greedy_chain(tgt, p, wl.max_new)
+    pk = wl.d + 5
+    assert len({g[0], g[1], g[pk - 1]}) == 3 and g[pk - 1] not in g[:pk - 1]
+    s = make_setup(wl, keywords=np.array([[g[0], g[1], g[pk - 1]]], np.int32),
+                   draft_equals_target=True)
+    eng, states, rep, adopted, n = run_parity(s, steps=12, tol=TOL32, tol_r=TOL32,
+                                              step1_budget=2)
+    tokens_match(eng, states)
+    assert states[0].T == g
+    assert rep.get("round2_ok", 0) == 1 and rep.get("round2", 0) == 4, rep
+
+
+def test_tiny_step1_budget2_mixed_states():
+    """b = 2 with independent models and keywords from M_p's greedy continuation: round 1,
+    round 2 and Step-2 each decide some S2/S3 steps; GPU and oracle agree step by step
+    (tokens and reward of every round 2 included)."""
+    wl = synth.scaled(synth.TINY, batch=2, max_new=24, r_t=0.6)
+    t_host = synth.model_weights(wl, "target", device="host")
+    tgt = oracle.Transformer(wl.target, t_host)
+    p = synth.prompts(wl)
+    kw = np.stack([np.array(greedy_chain(tgt, p[b].tolist(), 12)[2:12:4], np.int32)
+                   for b in range(wl.batch)])
+    s = make_setup(wl, keywords=kw)
+    eng, states, rep, adopted, n = run_parity(s, steps=24, tol=TOL32, tol_r=TOL32,
+                                              step1_budget=2)
+    tokens_match(eng, states)
+    print("budget-2 report:", rep)
+    assert rep.get("round2", 0) > 0, rep
+
+
+def test_tiny_step1_budget2_reward_head():
+    """b = 2 with the composite reward (coverage and the sigmoid head on M_p's hidden state):
+    round 2's reward takes the head at lh_d from the round's own target pass; r_t sits where
+    one covered keyword plus the head decides, so all outcomes occur."""
+    wl = synth.scaled(synth.TINY, batch=2, max_new=20, r_t=0.42, reward_head=True)
+    t_host = synth.model_weights(wl, "target", device="host")
+    tgt = oracle.Transformer(wl.target, t_host)
+    p = synth.prompts(wl)
+    kw = np.stack([np.array(greedy_chain(tgt, p[b].tolist(), 12)[1:12:4], np.int32)
+                   for b in range(wl.batch)])
+    s = make_setup(wl, keywords=kw)
+    eng, states, rep, adopted, n = run_parity(s, steps=20, tol=TOL32, tol_r=TOL32,
+                                              step1_budget=2)
+    tokens_match(eng, states)
+    print("budget-2 head report:", rep)
+    assert rep.get("round2", 0) > 0, rep
+
+
+def test_small_bf16_step1_budget2():
+    """b = 2 on the bf16 path (12-layer target, 4-layer draft, 8 prompts)."""
+    wl = synth.scaled(synth.SMALL, max_new=10)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=10, tol=TOL16, tol_r=TOL16,
+                                              step1_budget=2)
+    tokens_match(eng, states)
+    print("small budget-2 report:", rep, "adopted:", len(adopted))
+
+
 def test_tiny_cdlh_appx_on_the_same_kernels():
     """Alg. 2 CDLH-appx on the GPU path: M_q's lookaheads are never accepted (a_t, r_t above
     any score), so every step emits c_{b*}: the CDLH-appx token of the oracle's Alg. 2 with
