@@ -270,8 +270,10 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         s[q][1] += qv.x * k1.x + qv.y * k1.y + qv.z * k1.z + qv.w * k1.w;
       }
     }
-    // ---- online softmax: running max, rescale of l and o, probabilities of this chunk
-    float p0[QPW], p1[QPW];
+    // ---- online softmax: running max, rescale of l and o, probabilities of this chunk;
+    //      every stage runs over all QPW query vectors, so their shuffles are in flight
+    //      together (the same butterflies as warp_max / warp_sum)
+    float p0[QPW], p1[QPW], mx[QPW], alpha[QPW];
 #pragma unroll
     for (int q = 0; q < QPW; ++q) {
       const int qi = q0 + q;
@@ -287,19 +289,36 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         ok0 = s_kslot[k0] >= 0 && s_ktb[k0] == tb && s_kj[k0] < nt;
         ok1 = s_kslot[k1] >= 0 && s_ktb[k1] == tb && s_kj[k1] < nt;
       }
-      const float a0 = ok0 ? s[q][0] : -INFINITY, a1 = ok1 ? s[q][1] : -INFINITY;
-      const float m_new = fmaxf(m_run[q], warp_max(fmaxf(a0, a1)));
-      float alpha = 1.f;
+      s[q][0] = ok0 ? s[q][0] : -INFINITY;   // masked keys: exp(-inf - m) = 0 below
+      s[q][1] = ok1 ? s[q][1] : -INFINITY;
+      mx[q] = fmaxf(s[q][0], s[q][1]);
+    }
+#pragma unroll
+    for (int o2 = 16; o2 > 0; o2 >>= 1)
+#pragma unroll
+      for (int q = 0; q < QPW; ++q) mx[q] = fmaxf(mx[q], __shfl_xor_sync(0xffffffffu, mx[q], o2));
+#pragma unroll
+    for (int q = 0; q < QPW; ++q) {
+      const float m_new = fmaxf(m_run[q], mx[q]);
+      alpha[q] = 1.f;
       p0[q] = p1[q] = 0.f;
       if (m_new > -INFINITY) {
-        alpha = (m_run[q] > -INFINITY) ? expf(m_run[q] - m_new) : 0.f;
-        p0[q] = ok0 ? expf(a0 - m_new) : 0.f;
-        p1[q] = ok1 ? expf(a1 - m_new) : 0.f;
+        alpha[q] = (m_run[q] > -INFINITY) ? expf(m_run[q] - m_new) : 0.f;
+        p0[q] = expf(s[q][0] - m_new);
+        p1[q] = expf(s[q][1] - m_new);
       }
-      l_run[q] = alpha * l_run[q] + warp_sum(p0[q] + p1[q]);
       m_run[q] = m_new;
+      mx[q] = p0[q] + p1[q];   // from here: this lane's share of the sum
+    }
 #pragma unroll
-      for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] *= alpha;
+    for (int o2 = 16; o2 > 0; o2 >>= 1)
+#pragma unroll
+      for (int q = 0; q < QPW; ++q) mx[q] += __shfl_xor_sync(0xffffffffu, mx[q], o2);
+#pragma unroll
+    for (int q = 0; q < QPW; ++q) {
+      l_run[q] = alpha[q] * l_run[q] + mx[q];
+#pragma unroll
+      for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] *= alpha[q];
     }
     if constexpr (QPW == 4) {
       *reinterpret_cast<float4*>(pS + lane * L::PP + q0) = make_float4(p0[0], p0[1], p0[2], p0[3]);
@@ -368,19 +387,9 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   // ---- merge: block cx finishes query vectors cx, cx + C, ... (a warp per query vector),
   //      reading the C partials through distributed shared memory, 8 blocks at a time
   for (int qi = cx + warp * C; qi < nq; qi += C * AWARPS) {
-    float mr = -INFINITY, lr = 0.f;
-    if (lane < C) {
-      mr = cluster.map_shared_rank(s_pm, lane)[qi];
-      lr = cluster.map_shared_rank(s_pl, lane)[qi];
-    }
-    const float M = warp_max(mr);
-    const float w = (lane < C && mr > -INFINITY) ? expf(mr - M) : 0.f;
-    const float Lsum = warp_sum(w * lr);
-    float acc[DPL];
-#pragma unroll
-    for (int c2 = 0; c2 < DPL; ++c2) acc[c2] = 0.f;
-    for (int r0 = 0; r0 < C; r0 += 8) {
-      float vv[8][DPL];
+    // the first 8 blocks' partial o go out with (m, l): one round trip for C <= 8
+    float vv[8][DPL];
+    auto load_o = [&](int r0) {
 #pragma unroll
       for (int r = 0; r < 8; ++r) {
 #pragma unroll
@@ -396,6 +405,21 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
           }
         }
       }
+    };
+    load_o(0);
+    float mr = -INFINITY, lr = 0.f;
+    if (lane < C) {
+      mr = cluster.map_shared_rank(s_pm, lane)[qi];
+      lr = cluster.map_shared_rank(s_pl, lane)[qi];
+    }
+    const float M = warp_max(mr);
+    const float w = (lane < C && mr > -INFINITY) ? expf(mr - M) : 0.f;
+    const float Lsum = warp_sum(w * lr);
+    float acc[DPL];
+#pragma unroll
+    for (int c2 = 0; c2 < DPL; ++c2) acc[c2] = 0.f;
+    for (int r0 = 0; r0 < C; r0 += 8) {
+      if (r0 > 0) load_o(r0);
 #pragma unroll
       for (int r = 0; r < 8; ++r) {
         const float wr = __shfl_sync(0xffffffffu, w, (r0 + r) & 31);
