@@ -357,13 +357,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---- cluster split-K reduction: rank r sums rows [r*R/SK, (r+1)*R/SK) of the SK partial
     //      tiles in rank order (distributed shared memory) into a free pipeline stage and runs
     //      the epilogue on them
+    // the epilogue warps agree on whether the block gave up (the two named barriers below
+    // must be reached by all of them or by none)
+    const bool gave_up = warp >= 2 ? tc::named_barrier_or(1, kEpThreads, s_abort != 0) : true;
     tc::cluster_arrive();               // this block's partial tile is complete (release)
     tc::cluster_wait();                 // every block's is (acquire)
-    if (warp >= 2 && !s_abort) {
+    const bool reduce = warp >= 2 && !gave_up;
+    const int R = min(a.R, NP), r = c % SK, t = c / SK;
+    const int ra = r * R / SK, rb = (r + 1) * R / SK;
+    float* red = reinterpret_cast<float*>(smem);   // stage 0 (idle): [rb - ra][kTileLd]
+    if (reduce) {
       const int etid = threadIdx.x - 64;
-      const int R = min(a.R, NP), r = c % SK, t = c / SK;
-      const int ra = r * R / SK, rb = (r + 1) * R / SK;
-      float* red = reinterpret_cast<float*>(smem);   // stage 0 (idle): [rb - ra][kTileLd]
       const uint32_t tile_s = tc::smem_u32(tileS);
       for (int i = etid; i < (rb - ra) * 32; i += kEpThreads) {
         const uint32_t off = ((ra + (i >> 5)) * kTileLd + (i & 31) * 4) * 4;
@@ -374,12 +378,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         *reinterpret_cast<float4*>(red + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
       }
+    }
+    // this block has read the others' tiles (the sums above consumed every load): the
+    // barrier's second phase runs while the epilogue writes
+    tc::cluster_arrive();
+    if (reduce) {
+      const int etid = threadIdx.x - 64;
       tc::named_barrier(1, kEpThreads);
       if (rb > ra)
         tile_epilogue<__nv_bfloat16>(a, t * 128, ra, rb - ra, red, kTileLd, s_rs + ra, etid,
                                      kEpThreads);
     }
-    tc::cluster_arrive_relaxed();       // this block has read the others' tiles
     tc::cluster_wait();                 // no block leaves while its tile may still be read
   }
   tc::tc_fence_before();

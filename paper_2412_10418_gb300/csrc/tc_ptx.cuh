@@ -71,6 +71,21 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* m, uint32_t parity, int32_t*
   return true;
 }
 
+// Barrier among `nthreads` threads under hardware barrier `id` that also ORs a predicate
+// over them: every participant gets the same result.
+__device__ __forceinline__ bool named_barrier_or(int id, int nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, %2, %3, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
 // ------------------------------------------------------------------------------ cluster
 // Split cluster barrier: every thread of every block of the cluster arrives, then waits for
 // the phase. A relaxed arrive orders nothing; the default arrive releases this thread's prior
