@@ -50,6 +50,15 @@ def test_7b_shapes_bench_configuration():
     check(synth.SEVEN_B_SLICE, steps=3)
 
 
+def test_7b_full_depth_bench_configuration():
+    """The whole 7B workload as bench.py times it (32-layer target, 16-layer draft, the
+    512-token prompt, k = 4, d = 4), two steps (the second over the first one's committed
+    K/V): prefill roots, draft tokens and log q, every verify logit (bf16 error accumulated
+    over all 32 layers, still within 2e-2: measured 2.6e-4), n_b, the rewards, b*, the state
+    and the emission against the oracle at full depth."""
+    check(synth.SEVEN_B, steps=2)
+
+
 def test_13b_shapes_bench_configuration():
     """13B-shaped target (GQA 40/8, FFN 13824) with the 1B-shaped draft, 4 prompts of 1024
     tokens, k = 8, d = 6: 224 verify rows (two MMAs per K step: hi and lo no longer fit one)."""
