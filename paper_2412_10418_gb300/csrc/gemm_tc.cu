@@ -448,13 +448,15 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   const int cap = per_sm * n_sm * 87 / 100;
   // (the whole partial tile, n_pad rows, stays in shared memory: two stages must still fit)
   const bool tile_fits = fit(budget, p.n_pad) >= 2;
-  // Up to 12 blocks per tile while the grid stays within 192 blocks (measured, 7B draft
-  // down projection 2048 x 5504, 16 tiles: 8.43 us at 12 against 9.02 us at 8; larger
-  // non-portable clusters or grids lose, e.g. 16 x 16 blocks: 14.3 us).
+  // Up to 12 blocks per tile while the grid stays within 64 % of the block slots (measured
+  // at two blocks per SM, 7B draft down projection 2048 x 5504, 16 tiles: 8.43 us at 12
+  // blocks against 9.02 us at 8; larger non-portable clusters or grids lose, e.g. 16 x 16
+  // blocks: 14.3 us).
+  const int wide = per_sm * n_sm * 64 / 100;
   int S = cluster;
   if (S < 0)
     S = (tile_fits && 2 * p.tiles <= cap)
-            ? std::max(std::min(8, cap / p.tiles), std::min(12, 192 / p.tiles))
+            ? std::max(std::min(8, cap / p.tiles), std::min(12, wide / p.tiles))
             : 0;
   S = std::min(std::min(S, p.kb_total), g_max_cluster);
   if (S >= 2 && tile_fits) {
