@@ -357,6 +357,30 @@ def cpu_baseline(wl, tw, dw, tokens_per_step, n_layers):
                        f"depth; {tokens_per_step:.2f} tokens/step as measured on the GPU")}
 
 
+# ------------------------------------------------------------------------------ ranks
+
+def aggregate_ranks(total_ms, tokens, device="cpu"):
+    """Whole-job numbers over the ranks of the default process group: the slowest rank's
+    time and the tokens of all ranks (replicas: every rank decodes the whole workload on its
+    own GPU, nothing is exchanged on the data path)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(total_ms), float(tokens)], device=device, dtype=torch.float64)
+    mx = t.clone()
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(mx[0]), float(t[1])
+
+
+def sum_over_ranks(x, device="cpu"):
+    """A per-rank rate summed over the ranks (the end-to-end tokens/s of the replicas)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], device=device, dtype=torch.float64)
+    dist.all_reduce(t)
+    return float(t[0])
+
+
 # ------------------------------------------------------------------------------ main
 
 def gpu_main(args):
@@ -384,11 +408,7 @@ def gpu_main(args):
     total_ms, tokens = timed_steps(eng, wl, args.steps, args.warmup)
     clk = clocks.stop()
     if world > 1:
-        t = torch.tensor([total_ms, float(tokens)], device=device, dtype=torch.float64)
-        mx = t.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        total_ms, tokens = float(mx[0]), float(t[1])
+        total_ms, tokens = aggregate_ranks(total_ms, tokens, device)
     value = tokens / (total_ms / 1000.0)
     counters = eng.counters()
     launches_per_step = counters[6]
@@ -423,9 +443,7 @@ def gpu_main(args):
     if not args.no_e2e:
         ev, h2d, d2h, n_e2e = e2e_run(eng, wl, args.steps)
         if world > 1:
-            t = torch.tensor([ev], device=device, dtype=torch.float64)
-            dist.all_reduce(t)
-            ev = float(t[0])
+            ev = sum_over_ranks(ev, device)
         e2e = {"value": round(ev, 3), "unit": "tokens/s", "h2d_bytes_per_step": round(h2d, 1),
                "d2h_bytes_per_step": d2h,
                "note": f"whole generations: pinned prompts+keywords in, prefill, then {n_e2e} "
