@@ -442,7 +442,7 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   const long long units = (long long)p.tiles * p.kb_total;
   p.ctas = (int)std::min<long long>(std::min<long long>(units, (long long)per_sm * n_sm),
                                     (long long)p.tiles * (max_split > 0 ? max_split : kMaxSplit));
-  // few tiles: a cluster of S <= 8 blocks per tile, all tiles resident at once. Clusters are
+  // few tiles: a cluster of S <= 12 blocks per tile, all tiles resident at once. Clusters are
   // placed whole within a GPC; on 152 SMs at two blocks each, grids of clusters past ~87 % of
   // the block slots no longer fit in one wave (measured), hence the cap.
   const int cap = per_sm * n_sm * 87 / 100;
