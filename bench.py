@@ -438,6 +438,14 @@ def gpu_main(args):
                         "frac": round(b / (ms / n / 1000.0) / 1e9 / hbm, 3)}
                        for b, (n, ms) in shapes.items()), key=lambda r: -r["avg_us"] * r["launches"])
     roofline["by_shape"] = by_shape[:8]
+    # the same bytes over the graph-replayed step (everything else in the step included): a
+    # lower bound on the projections' rate inside the CUDA graph
+    step_bytes = dom[1]["bytes"] / n_prof
+    step_ms = total_ms / args.steps   # every rank times args.steps steps; the slowest rank
+    roofline["in_graph_lower_bound"] = {
+        "bytes_per_step": round(step_bytes), "ms_per_step": round(step_ms, 4),
+        "GB/s": round(step_bytes / (step_ms / 1000.0) / 1e9, 1),
+        "frac": round(step_bytes / (step_ms / 1000.0) / 1e9 / hbm, 4)}
     verify_bytes = (wl.target.n_params() * 2)
     e2e = None
     if not args.no_e2e:
