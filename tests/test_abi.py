@@ -125,3 +125,19 @@ def test_init_rejects_before_touching_the_device(cdsl):
                          1 << 20, 1 << 30, None, ctypes.byref(ctx))
     assert code == 1 and "reward" in cdsl.cdsl_last_error(None)
     assert ctx.value is None
+
+
+def test_step1_budget_2_adds_the_round_buffers(cdsl):
+    """Budget 2 carves the Step-1 round's KV tail regions (d+2 target and d+1 draft slots per
+    prompt, every layer) and its d+2-row target pass on top of budget 1."""
+    wl = synth.scaled(synth.TINY, k=1)   # one beam: the round's d+2 rows exceed the d+1 verify rows
+    t, d, r1 = cfgs(cdsl, wl, step1_budget=1)
+    _, _, r2 = cfgs(cdsl, wl, step1_budget=2)
+    n1, n2 = cdsl.cdsl_workspace_size(t, d, r1), cdsl.cdsl_workspace_size(t, d, r2)
+    tails = 4 * 2 * (wl.target.n_layers * (wl.d + 2) * wl.target.n_kv_heads * wl.target.head_dim
+                     + wl.draft.n_layers * (wl.d + 1) * wl.draft.n_kv_heads * wl.draft.head_dim)
+    assert n2 - n1 >= tails * wl.batch
+
+
+def test_get_step1_needs_a_context(cdsl):
+    assert cdsl.lib().cdsl_get_step1(None, None, None, None) == 1   # CDSL_EINVAL
