@@ -84,6 +84,16 @@ def test_beam_and_lookahead_extremes(k, d):
     tokens_match(eng, states)
 
 
+def test_tiny_maximum_context():
+    """The longest context the attention takes (8128 positions): an 8100-token prompt, so the
+    passes see 127 prefix chunks of 64 keys plus the beam tails, 8 chunks per block of a
+    16-block cluster; the prefill runs 127 passes of 64 rows."""
+    wl = synth.scaled(synth.TINY, prompt_len=8100, max_new=8, k=2, d=2)
+    s = make_setup(wl)
+    eng, states, rep, adopted, n = run_parity(s, steps=4, tol=TOL32, tol_r=TOL32)
+    tokens_match(eng, states)
+
+
 def test_graph_step_equals_separate_calls():
     import torch
     wl = synth.scaled(synth.TINY, batch=2, max_new=12)
