@@ -68,9 +68,17 @@ def config_of(wl):
         "batch": wl.batch, "prompt_len": wl.prompt_len, "k": wl.k, "d": wl.d,
         "max_new": wl.max_new, "a_t": wl.a_t, "r_t": wl.r_t,
         "reward": "0.5*coverage+0.5*sigmoid(w.h)" if wl.reward_head else "coverage",
-        "l2": f"inputs larger than L2: every step streams all weights "
-              f"({(wl.target.n_params() + wl.d * wl.draft.n_params()) * 2 / 1e9:.1f} GB)",
+        "l2": f"inputs larger than L2: every step streams every projection and LM-head "
+              f"weight ({streamed_weight_bytes(wl) / 1e9:.1f} GB; the embeddings are gathered)",
     }
+
+
+def streamed_weight_bytes(wl):
+    """Weight bytes one step reads through the projections: the target once, the draft once
+    per lookahead call (every matrix but the embedding table, whose rows are gathered)."""
+    def per_model(m):
+        return sum(math.prod(s) for n, s in m.weight_specs() if n != "embed") * 2
+    return per_model(wl.target) + wl.d * per_model(wl.draft)
 
 
 def gemm_traffic_ratio():
