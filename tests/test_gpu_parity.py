@@ -306,6 +306,22 @@ def test_tiny_step1_budget2_reward_head():
     assert rep.get("round2", 0) > 0, rep
 
 
+def test_tiny_speculative_sampling_with_step1_budget2():
+    """Speculative-sampling validation (f1) together with the Step-1 budget b = 2 (f2): the
+    acceptance counts come from the draws, round 2 from the verify row of beam 1."""
+    wl = synth.scaled(synth.TINY, batch=2, max_new=16, r_t=0.6)
+    t_host = synth.model_weights(wl, "target", device="host")
+    tgt = oracle.Transformer(wl.target, t_host)
+    p = synth.prompts(wl)
+    kw = np.stack([np.array(greedy_chain(tgt, p[b].tolist(), 12)[2:12:4], np.int32)
+                   for b in range(wl.batch)])
+    s = make_setup(wl, keywords=kw)
+    eng, states, rep, adopted, n = run_parity(s, steps=16, tol=TOL32, tol_r=TOL32,
+                                              acceptance=1, seed=11, step1_budget=2)
+    tokens_match(eng, states)
+    print("speculative + budget-2 report:", rep)
+
+
 def test_small_bf16_step1_budget2():
     """b = 2 on the bf16 path (12-layer target, 4-layer draft, 8 prompts)."""
     wl = synth.scaled(synth.SMALL, max_new=10)
