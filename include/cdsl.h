@@ -91,17 +91,18 @@ typedef struct cdsl_run_cfg {
   int32_t reward_head;  /* 0: R = coverage; 1: R = 0.5 coverage + 0.5 sigmoid(w . h_last) */
   int32_t page_size;    /* KV page size in tokens (power of two, 16..256); 0 = 64 */
   int32_t max_chunk;    /* rows per prefill forward pass; 0 = 64 */
-  /* Validation of the lookahead by M_p (Sec. 3.2.2, P:125-131):
+  /* Validation of the lookahead by M_p (Sec. 3.2.2):
    *   0: hard rejection: x_j is accepted while argmax p_j == x_j;
    *   1: speculative sampling: x_j is accepted while u_j <= min(1, p_j(x_j) / q_j(x_j)),
    *      tested as log(u_j) <= log p_j(x_j) - log q_j(x_j) in float32. The rejected position's
-   *      resampled token is never emitted, so only the count n_b is used.
+   *      resampled token is never emitted (CDSL keeps only accepted drafts, Sec. 3.2.2), so
+   *      only the count n_b is used.
    * u_j = (SplitMix64 output number c of the generator seeded with `seed`) >> 40, times 2^-24,
    * where c = ((step * batch + b) * k + beam) * d + (j - 1) and step counts the completed
    * steps of the context (SplitMix64: Steele, Lea, Flood, OOPSLA 2014). */
   int32_t acceptance;
   uint32_t seed;
-  /* Step-1 budget b of Alg. 1's S2/S3 branch (P:176-190, Sec. 3.2.3), 0, 1 or 2. With b >= 1,
+  /* Step-1 budget b of Alg. 1's S2/S3 branch (Sec. 3.2.3), 0, 1 or 2. With b >= 1,
    * a step in S2/S3 (a < a_t) first tries M_p's greedy token, the root c_1, whose draft
    * lookahead and reward r_1^full the step already has: if r_1^full >= r_t it emits c_1
    * (state 3) instead of the CDLH-appx token c_{b*} of Step-2. With b = 2, when that fails,
@@ -211,7 +212,7 @@ CDSL_API int32_t cdsl_get_profile(cdsl_ctx* ctx, int32_t impl, double* h_out);
  * the stream. */
 CDSL_API int32_t cdsl_get_profile_launches(cdsl_ctx* ctx, double* h_out, int32_t h_capacity);
 
-/* Step-1 round 2 of the last cdsl_select / cdsl_step (budget 2; Alg. 1): d_need [B]
+/* Step-1 round 2 of the last cdsl_select / cdsl_step (budget 2; Alg. 1, S2/S3 Step-1): d_need [B]
  * 1 where round 1 failed in S2/S3 so that round 2 decided the step, d_tokens [B, d+1] the
  * round's x' and lookahead lh_1..lh_d, d_reward [B] R(T + c_1 + x' + lh) (meaningful where
  * d_need = 1). Any pointer may be NULL. CDSL_EINVAL with a smaller budget. */
@@ -221,21 +222,25 @@ CDSL_API int32_t cdsl_get_step1(cdsl_ctx* ctx, int32_t* d_need, int32_t* d_token
  * device-side error was latched) in *h_device_status. Clears nothing. */
 CDSL_API int32_t cdsl_get_status(cdsl_ctx* ctx, int32_t* h_device_status);
 
-/* Weight-streaming GEMM that allocates nothing (the paper has no counterpart; it serves
- * callers of this library that cannot allocate device memory: code running while a stream
- * is captured in global mode, where cudaMalloc is an error; host frameworks whose own
- * allocator holds the GPU's memory; latency-critical loops that must not block on the
- * allocator). y[R, N] = x[R, K] W^T, fp32 accumulation, computed by the split-K kernel of
- * the draft calls: d_w [N, K] bfloat16 row-major, d_x [R, K] float32, d_y [R, N] float32,
- * all device pointers, 16-byte aligned; stream is a cudaStream_t (NULL: legacy stream).
- * Limits: 1 <= R <= 8, 8 <= K <= 8192 with K % 8 == 0, 1 <= N <= 32768; anything beyond
- * them returns CDSL_EINVAL without launching. Its scratch (split-K partials, arrival counters
- * and the hi/lo activation planes, 8.3 MiB) is one fixed array inside the library that every
- * GPU loading the library holds until the process exits; no call allocates or frees memory.
- * The first call on a device looks up that array's address (and clears its counters) with
- * the device current, so make that first call before any stream capture. Every call reuses
- * the same array: calls that overlap on a GPU (other streams or threads) race, and the caller
- * must order them. Asynchronous on `stream`; errors via cdsl_last_error(NULL). */
+/* Weight-streaming GEMM that allocates nothing (the paper has no counterpart). It serves
+ * callers of this library that cannot allocate device memory: host frameworks whose own
+ * caching allocator has already reserved the GPU's memory, real-time loops that must not
+ * block on cudaMalloc / cudaFree, and runtimes that forbid device allocation after start-up.
+ * y[R, N] = x[R, K] W^T with fp32 accumulation, computed by the library's CUDA-core split-K
+ * GEMV (x is split into bf16 hi and lo planes, so the result is within about 1e-5 relative
+ * of the exact product): d_w [N, K] bfloat16 row-major, d_x [R, K] float32, d_y [R, N]
+ * float32, all device pointers on the current device, contiguous and 16-byte aligned; stream
+ * is a cudaStream_t (NULL: the legacy stream).
+ * Limits: 1 <= R <= 8, 8 <= K <= 8192 with K % 8 == 0, 1 <= N <= 32768; anything beyond them
+ * returns CDSL_EINVAL without launching. Its scratch (split-K partials, arrival counters and
+ * the hi/lo activation planes, 8.3 MiB) is one fixed array inside the library, which every
+ * GPU that loads the library holds until the process exits; no call allocates or frees.
+ * Set-up: the first call in each CUDA context looks up that array's device address (and
+ * clears its counters) with the context current, so make that first call before any stream
+ * capture. Only contexts that stay alive are supported: after a device reset the array's
+ * address may be stale. Every call shares the array: calls that overlap on a GPU (other
+ * streams or threads) race, and the caller must order them. Asynchronous on `stream`;
+ * errors via cdsl_last_error(NULL). */
 CDSL_API int32_t cdsl_gemv_noalloc(const void* d_w, int32_t N, int32_t K, const float* d_x,
                                    int32_t R, float* d_y, void* stream);
 

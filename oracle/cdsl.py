@@ -63,6 +63,9 @@ class Decider:
         self.tol = tol
         self.tol_r = tol_r
         self.adopted: List[tuple] = []
+        # the oracle's own margin against each adopted choice, in the units of its tolerance
+        # (logit / log-probability / reward differences), in the order of ``adopted``
+        self.margins: List[float] = []
 
     def _theirs(self, kind, idx):
         if self.other is None or kind not in self.other:
@@ -76,6 +79,7 @@ class Decider:
             g = int(g)
             if g != a and 0 <= g < v.shape[0] and v[g] != v[a] and v[g] >= v[a] - self.tol:
                 self.adopted.append((kind, idx, a, g))
+                self.margins.append(float(v[a] - v[g]))
                 return g
         return a
 
@@ -89,6 +93,7 @@ class Decider:
                     and np.all(np.abs(v[g] - v[order]) <= self.tol)
                     and not np.all(v[g] == v[order])):
                 self.adopted.append((kind, idx, order.tolist(), g.tolist()))
+                self.margins.append(float(np.max(np.abs(v[g] - v[order]))))
                 return g
         return order
 
@@ -102,6 +107,7 @@ class Decider:
             g = int(g)
             if g != best and r[g] != best_r and r[g] >= best_r - self.tol_r:
                 self.adopted.append((kind, idx, best, g))
+                self.margins.append(float(best_r - r[g]))
                 return g
         return best
 
@@ -116,6 +122,7 @@ class Decider:
             theirs = j < int(g)
             if theirs != ok and abs(log_u - log_ratio) <= self.tol:
                 self.adopted.append((kind, idx, j, ok, theirs))
+                self.margins.append(float(abs(log_u - log_ratio)))
                 return theirs
         return ok
 
@@ -125,6 +132,7 @@ class Decider:
         g = self._theirs(kind, idx)
         if g is not None and abs(r - r_t) <= self.tol_r and bool(g) != ok:
             self.adopted.append((kind, idx, ok, bool(g)))
+            self.margins.append(float(abs(r - r_t)))
             return bool(g)
         return ok
 
@@ -500,7 +508,7 @@ def cdlh_token(target: Transformer, lookahead: Transformer, st: PromptState,
     the largest R(pfx + x_i + lh) wins (strict '>', so the first of equal rewards).
 
     Reading: the candidate x_i is part of the scored text and the prefix update happens once,
-    after the candidate loop (the listing's loop nesting and R(pfx + lh) are taken as typos)."""
+    after the candidate loop (Algorithm 2's loop nesting and its R(pfx + lh) are read as typos)."""
     if base:
         tcache, p, _ = _extend(target, st.tcache, base)
         p = p[-1]
@@ -532,7 +540,10 @@ def _commit(target, draft, st: PromptState, out: List[int], keep_draft_logits=Tr
 
 def alg1_step(target: Transformer, draft: Transformer, st: PromptState, run: RunParams,
               w_head) -> dict:
-    """One iteration of Algorithm 1's while-loop, as printed (hard rejection, budget b).
+    """One decision of literal Algorithm 1 (Sec. 3.2.3; hard rejection, Step-1 budget b), from the
+    method's description: d greedy M_q tokens, one M_p pass over them, the count n of accepted
+    tokens, the reward of the accepted span, then S1, S2/S3 (Step-1 rounds, else the Step-2
+    CDLH-appx token) or S4.
 
     Readings: the verify pass yields p_i = M_p(pfx + x_<i) for i = 1..d (its last row, the
     (d+1)-th distribution, is not used); Step-1 tokens are new tokens appended to X, the

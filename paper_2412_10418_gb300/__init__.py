@@ -20,6 +20,8 @@ LIB_PATH = os.path.join(HERE, "libcdsl_gb300.so")
 DTYPE_F32, DTYPE_BF16 = 0, 1
 STATUS = {0: "CDSL_OK", 1: "CDSL_EINVAL", 2: "CDSL_ENOMEM", 3: "CDSL_ECUDA", 4: "CDSL_ETIMEOUT",
           5: "CDSL_ENONFINITE", 6: "CDSL_ESTATE", 7: "CDSL_ERANGE"}
+(CDSL_OK, CDSL_EINVAL, CDSL_ENOMEM, CDSL_ECUDA, CDSL_ETIMEOUT, CDSL_ENONFINITE, CDSL_ESTATE,
+ CDSL_ERANGE) = range(8)
 S1, S2_S3, S4 = 1, 2, 4
 
 
@@ -217,9 +219,33 @@ def cdsl_get_profile_launches(ctx, capacity: int = 8192):
 
 def cdsl_gemv_noalloc(w, x, y, stream=None):
     """y[R, N] = x[R, K] w^T through the weight-streaming kernel with its scratch in a fixed
-    array inside the library (no device memory is allocated); see include/cdsl.h."""
+    array inside the library (no device memory is allocated); see include/cdsl.h.
+
+    The C ABI sees only pointers and sizes, so the shapes, dtypes, layouts and devices are
+    checked here: w bfloat16 [N, K], x float32 [R, K], y float32 [R, N], all contiguous and on
+    the current CUDA device. Anything else raises CdslError(CDSL_EINVAL) before the call."""
+    import torch
+
+    def bad(why):
+        raise CdslError(CDSL_EINVAL, "cdsl_gemv_noalloc: " + why)
+
+    ts = (w, x, y)
+    if not all(isinstance(t, torch.Tensor) for t in ts):
+        bad("w, x and y must be torch tensors")
+    if w.dtype != torch.bfloat16 or x.dtype != torch.float32 or y.dtype != torch.float32:
+        bad("w must be bfloat16, x and y float32")
+    if w.dim() != 2 or x.dim() != 2 or y.dim() != 2:
+        bad("w, x and y must be 2-D")
     N, K = w.shape
     R = x.shape[0]
+    if tuple(x.shape) != (R, K) or tuple(y.shape) != (R, N):
+        bad(f"shapes: w {tuple(w.shape)}, x {tuple(x.shape)}, y {tuple(y.shape)} "
+            "(want [N, K], [R, K], [R, N])")
+    if not all(t.is_contiguous() for t in ts):
+        bad("w, x and y must be contiguous")
+    dev = torch.cuda.current_device() if torch.cuda.is_available() else None
+    if not all(t.is_cuda and t.device.index == dev for t in ts):
+        bad("w, x and y must be on the current CUDA device")
     _check(lib().cdsl_gemv_noalloc(w.data_ptr(), N, K, x.data_ptr(), R, y.data_ptr(), stream))
 
 

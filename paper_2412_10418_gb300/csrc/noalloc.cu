@@ -1,18 +1,21 @@
 // noalloc.cu -- cdsl_gemv_noalloc: the weight-streaming GEMM for callers that cannot allocate.
 //
-// Some callers cannot hand this library a workspace: code that runs while a stream is being
-// captured in global capture mode (where cudaMalloc is an error), a host framework whose own
-// allocator has already reserved the GPU's memory, or a latency-critical loop that must not
-// block on cudaMalloc / cudaFree. For them this entry point runs the same split-K kernel the
-// draft calls use, with every byte of its scratch -- the hi/lo activation planes, the split-K
-// partial tiles and the per-tile arrival counters -- in one fixed device array below. The
-// array is created with the library's module on every GPU that loads it and lives until the
-// process exits; nothing is allocated per call.
+// Some callers cannot hand this library a workspace: a host framework whose own caching
+// allocator has already reserved the GPU's memory, a real-time loop that must not block on
+// cudaMalloc / cudaFree, a runtime that forbids device allocation after start-up. For them this
+// entry point runs the CUDA-core split-K GEMV (gemv_stream.cu) with every byte of its scratch --
+// the hi/lo activation planes, the split-K partial tiles and the per-tile arrival counters --
+// in one fixed device array below. The array is created with the library's module on every GPU
+// that loads it and lives until the process exits; nothing is allocated per call.
 //
 // Host code must not pass the array's name to a kernel: on the host that name is only a
-// stand-in symbol, not a device address. The device address is looked up once per device,
-// with that device current, by cudaGetSymbolAddress, and passed to the kernels.
+// stand-in symbol, not a device address. The device address is looked up once per CUDA
+// context, with that context current, by cudaGetSymbolAddress, and passed to the kernels.
+#include <cuda.h>
+
 #include <mutex>
+#include <utility>
+#include <vector>
 
 #include "gemm.cuh"
 #include "kernels.h"
@@ -35,9 +38,11 @@ constexpr size_t kScratchBytes = kPartBytes + kCntBytes + kPlaneBytes;
 
 static __device__ __align__(256) unsigned char g_gemv_scratch[kScratchBytes];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-unsigned char* g_scratch_dev[kMaxDevices] = {};
+// (context, device address of the array in it), one entry per context set up so far
+std::vector<std::pair<CUcontext, unsigned char*>> g_scratch_ctx;
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+CtxGetCurrentFn g_ctx_get_current = nullptr;
 
 // x [n] fp32 -> hi plane [n], lo plane [n] (the GEMM-input format of bf16 models)
 __global__ void k_split_planes(const float* x, int n, __nv_bfloat16* planes) {
@@ -45,28 +50,53 @@ __global__ void k_split_planes(const float* x, int n, __nv_bfloat16* planes) {
   if (i < n) store_act<__nv_bfloat16>(planes, (size_t)n, (size_t)i, x[i]);
 }
 
-// Device address of the scratch array on the current device (set-up on first use).
+// The current CUDA context (the runtime's primary context of the current device once a
+// runtime call has made it current); nullptr where none is current yet.
+CUcontext current_context() {
+  if (!g_ctx_get_current) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &fn, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn)
+      return nullptr;
+    g_ctx_get_current = reinterpret_cast<CtxGetCurrentFn>(fn);
+  }
+  CUcontext c = nullptr;
+  return g_ctx_get_current(&c) == CUDA_SUCCESS ? c : nullptr;
+}
+
+// Device address of the scratch array in the current context (set-up on first use there).
 int scratch_address(unsigned char** out, const char** why) {
   int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) {
     *why = "cdsl_gemv_noalloc: no usable current CUDA device";
     return CDSL_ECUDA;
   }
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_dev[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_gemv_scratch) != cudaSuccess || !p) {
-      *why = "cdsl_gemv_noalloc: cudaGetSymbolAddress of the scratch array failed";
-      return CDSL_ECUDA;
+  CUcontext ctx = current_context();
+  for (const auto& e : g_scratch_ctx)
+    if (ctx && e.first == ctx) {
+      *out = e.second;
+      return CDSL_OK;
     }
-    // the arrival counters must start at zero (each launch leaves them at zero again)
-    if (cudaMemset(static_cast<unsigned char*>(p) + kPartBytes, 0, kCntBytes) != cudaSuccess) {
-      *why = "cdsl_gemv_noalloc: clearing the arrival counters failed";
-      return CDSL_ECUDA;
-    }
-    g_scratch_dev[dev] = static_cast<unsigned char*>(p);
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_gemv_scratch) != cudaSuccess || !p) {
+    *why = "cdsl_gemv_noalloc: cudaGetSymbolAddress of the scratch array failed";
+    return CDSL_ECUDA;
   }
-  *out = g_scratch_dev[dev];
+  ctx = current_context();   // the lookup above made the device's primary context current
+  if (!ctx) {
+    *why = "cdsl_gemv_noalloc: no current CUDA context";
+    return CDSL_ECUDA;
+  }
+  // the arrival counters must start at zero (each launch leaves them at zero again)
+  if (cudaMemset(static_cast<unsigned char*>(p) + kPartBytes, 0, kCntBytes) != cudaSuccess) {
+    *why = "cdsl_gemv_noalloc: clearing the arrival counters failed";
+    return CDSL_ECUDA;
+  }
+  g_scratch_ctx.emplace_back(ctx, static_cast<unsigned char*>(p));
+  *out = static_cast<unsigned char*>(p);
   return CDSL_OK;
 }
 

@@ -141,3 +141,40 @@ def test_step1_budget_2_adds_the_round_buffers(cdsl):
 
 def test_get_step1_needs_a_context(cdsl):
     assert cdsl.lib().cdsl_get_step1(None, None, None, None) == 1   # CDSL_EINVAL
+
+
+@pytest.mark.parametrize("R,K,N,offset", [
+    (0, 768, 32000, 0),       # no rows
+    (9, 768, 32000, 0),       # more rows than the fixed scratch holds
+    (4, 8200, 1000, 0),       # K beyond 8192
+    (4, 4, 1000, 0),          # K below 8
+    (4, 772, 1000, 0),        # K not a multiple of 8
+    (4, 768, 0, 0),           # no outputs
+    (4, 768, 32769, 0),       # N beyond 32768
+    (4, 768, 1000, 8),        # misaligned pointers
+])
+def test_gemv_noalloc_rejects_before_any_cuda_call(cdsl, R, K, N, offset):
+    """Sizes beyond the fixed scratch and misaligned pointers return CDSL_EINVAL from the
+    host-side checks, before the library touches CUDA (the pointers are never dereferenced)."""
+    lib = cdsl.lib()
+    base = 1 << 20
+    rc = lib.cdsl_gemv_noalloc(base + offset, N, K, base + 4096 + offset, R,
+                               base + 8192 + offset, None)
+    assert rc == cdsl.CDSL_EINVAL
+    assert "cdsl_gemv_noalloc" in cdsl.cdsl_last_error(None)
+    assert lib.cdsl_gemv_noalloc(None, 1000, 768, base, 4, base, None) == cdsl.CDSL_EINVAL
+
+
+def test_gemv_noalloc_binding_checks_tensors(cdsl):
+    """The binding refuses dtypes, shapes, layouts and devices the C ABI cannot check."""
+    import torch
+    w = torch.zeros((64, 32), dtype=torch.bfloat16)
+    x = torch.zeros((2, 32), dtype=torch.float32)
+    y = torch.zeros((2, 64), dtype=torch.float32)
+    cases = [(w.float(), x, y, "bfloat16"), (w, x.double(), y, "float32"),
+             (w, torch.zeros((2, 16)), y, "shapes"), (w, x, torch.zeros((2, 63)), "shapes"),
+             (w, torch.zeros((32, 2)).t(), y, "contiguous"), (w, x, y, "CUDA device")]
+    for ww, xx, yy, msg in cases:
+        with pytest.raises(cdsl.CdslError) as e:
+            cdsl.cdsl_gemv_noalloc(ww, xx, yy)
+        assert e.value.code == cdsl.CDSL_EINVAL and msg in str(e.value), (msg, str(e.value))

@@ -119,7 +119,8 @@ def test_small_bf16_parity():
 
 @pytest.mark.parametrize("batch,k", [(1, 4), (2, 2), (1, 8)])
 def test_small_bf16_few_rows(batch, k):
-    """Draft calls with B*k (+B) <= 8 rows take the weight-streaming GEMM (split-K)."""
+    """Draft calls with B*k (+B) <= 8 rows: the tensor-core GEMM's cluster split-K schedules
+    at the smallest activation tile (16 rows, of which at most 8 are live)."""
     wl = synth.scaled(synth.SMALL, batch=batch, k=k, max_new=10)
     s = make_setup(wl)
     eng, states, rep, adopted, n = run_parity(s, steps=4, tol=TOL16, tol_r=TOL16)
@@ -128,8 +129,8 @@ def test_small_bf16_few_rows(batch, k):
 
 
 def test_small_bf16_forced_acceptance():
-    """bf16, draft := target, B = 1: full acceptance and S1 emissions through the
-    weight-streaming path, including the pending draft row of the next step."""
+    """bf16, draft := target, B = 1: full acceptance and S1 emissions (multi-token commits),
+    including the pending draft row of the next step's first draft call."""
     wl = synth.scaled(synth.SMALL, batch=1, draft=synth.SMALL.target, max_new=16, n_keywords=3)
     s = make_setup(wl, draft_equals_target=True)
     tgt = oracle.Transformer(wl.target, s.t_host)

@@ -62,6 +62,58 @@ def test_reward_cases():
     assert reward(kws, [3], h, w, True) == pytest.approx(0.5 * (1 / 3) + 0.25)
 
 
+def test_reward_composite_away_from_zero():
+    """The composite reward's head term where w.h != 0, on closed forms: w.h = ln 3 gives a
+    sigmoid of exactly 3/4, w.h = -ln 3 exactly 1/4 (a flipped sign swaps the two), and a
+    large positive (negative) w.h drives the head term to 1 (0)."""
+    kws = [3, 4, 5, 6]
+    w = np.array([1.0, 2.0, 0.0])
+    h = np.array([1.0, 2.0, 7.0]) * (np.log(3.0) / 5.0)   # w.h = (1 + 4) ln 3 / 5 = ln 3
+    text = [3, 9, 5]                                      # 2 of 4 keywords: coverage 1/2
+    assert reward(kws, text, h, w, True) == pytest.approx(0.5 * 0.5 + 0.5 * 0.75, abs=1e-15)
+    assert reward(kws, text, -h, w, True) == pytest.approx(0.5 * 0.5 + 0.5 * 0.25, abs=1e-15)
+    assert reward(kws, [], h, w, True) == pytest.approx(0.375, abs=1e-15)
+    assert reward(kws, [], 40.0 * h, w, True) == pytest.approx(0.5, abs=1e-12)
+    assert reward(kws, [], -40.0 * h, w, True) == pytest.approx(0.0, abs=1e-12)
+
+
+def test_step_head_on_a_bigram_model():
+    """The per-row head term of a CDSL-k step and the composite rewards built from it, on a
+    target whose attention and FFN outputs are zero (Wo = W_down = 0): its final hidden state
+    at every position is then RMSNorm(E[token]) in closed form, so the head of verify row
+    (i, j) is sigmoid(w . RMSNorm(E[t_ij])) with t_i = [c_i, x_i1..x_id]. The weights w are
+    drawn so that the rows' w.h take both signs well away from 0."""
+    shp = shape(vocab=16)
+    rng = np.random.default_rng(21)
+    wt = {n: (np.ones(s, np.float32) if len(s) == 1 else
+              (0.5 * rng.standard_normal(s)).astype(np.float32)) for n, s in shp.weight_specs()}
+    for l in range(shp.n_layers):
+        wt[f"l{l}.wo"][:] = 0.0
+        wt[f"l{l}.w_down"][:] = 0.0
+    tgt = Transformer(shp, wt)
+    drf = model(shp, 22)
+    run = run_params(k=3, d=3, a_t=0.3, r_t=0.3, max_new=8, composite_reward=True)
+    w = 0.5 * np.random.default_rng(23).standard_normal(shp.d_model)
+    emb = wt["embed"].astype(np.float64)
+    hf = emb / np.sqrt(np.mean(emb * emb, axis=-1, keepdims=True) + shp.norm_eps)   # gain 1
+    z_tok = hf @ w                                     # w . h for every token id
+    assert z_tok.max() > 1.0 and z_tok.min() < -1.0
+    kw = [2, 5, 11]
+    st = prefill(tgt, drf, np.array([[1, 7, 3, 2]]), np.array([kw]))
+    for _ in range(2):
+        T0 = list(st[0].T)
+        rec = cdsl_k_step(tgt, drf, st, run, w)[0]
+        for i in range(run.k):
+            toks = [int(rec.roots[i])] + rec.x[i].tolist()
+            want = 1.0 / (1.0 + np.exp(-z_tok[toks]))
+            assert np.allclose(rec.head[i], want, rtol=0, atol=1e-9)
+            cov_full = coverage(kw, T0 + toks)
+            assert rec.r_full[i] == pytest.approx(0.5 * cov_full + 0.5 * want[run.d], abs=1e-9)
+            n = int(rec.n[i])
+            cov_acc = coverage(kw, T0 + toks[:n + 1])
+            assert rec.r_acc[i] == pytest.approx(0.5 * cov_acc + 0.5 * want[n], abs=1e-9)
+
+
 @pytest.mark.parametrize("d", [1, 2, 3, 4, 5, 6, 8, 10])
 @pytest.mark.parametrize("a_t", [0.0, 0.25, 0.3, 0.4, 0.5, 0.6, 0.8, 0.9, 1.0, 1.5])
 def test_n_min_is_exact_threshold(d, a_t):
@@ -558,3 +610,25 @@ def test_step1_rounds_match_literal_algorithm1(seed):
         assert rec.emitted == lit["emitted"]
         compared[0 if rec.state == S2_S3 else len(rec.emitted)] += 1
     assert min(compared.values()) >= 1   # Step-2, round-1 and round-2 outcomes all compared
+
+
+def test_adoption_bound_rejects_wide_margins():
+    """The parity harness fails a run where the oracle adopted a choice whose own margin is
+    wider than the bound (a wrong choice on the other side, not rounding), and passes one
+    within it."""
+    from cdsl_parity import adopt_bound_for, check_adoptions
+    bound = adopt_bound_for(2e-2)
+    assert bound == pytest.approx(3e-3) and adopt_bound_for(1e-4) == pytest.approx(1e-4)
+    logits = np.zeros((1, 1, 1, 4))
+    for gap, ok in ((1e-3, True), (5e-3, False)):
+        dec = Decider(other={"argmax": {(0, 0, 0): 2}}, tol=2e-2)
+        v = np.array([0.0, 1.0, 1.0 - gap, 0.5])
+        assert dec.argmax(v, "argmax", (0, 0, 0)) == 2 and dec.margins == [pytest.approx(gap)]
+        logits[0, 0, 0] = v
+        rep = {}
+        if ok:
+            check_adoptions(dec, {"logits": logits}, bound, rep)
+            assert rep["adopt_margin"] == pytest.approx(gap)
+        else:
+            with pytest.raises(AssertionError):
+                check_adoptions(dec, {"logits": logits}, bound, rep)

@@ -1,15 +1,19 @@
-"""cdsl_gemv_noalloc (the GEMM entry point that allocates no device memory) against the step
-library's own verify pass.
+"""cdsl_gemv_noalloc (the GEMM entry point that allocates no device memory) against an fp64
+product computed by torch, and against the step library's own verify pass.
 
-Some callers of this library cannot allocate device memory: code that runs while a stream is
-captured in global mode, host frameworks whose allocator already holds the GPU's memory, and
-latency-critical loops that must not block on cudaMalloc. cdsl_gemv_noalloc serves them: its
-scratch is a fixed array inside the library. This test builds a bf16 model whose layers leave
-the residual stream unchanged (the attention-output and FFN-down projections are zero), so
-cdsl_verify's logits are lm_head(RMSNorm(E[token])) for every verify row. It recomputes those
-normalized rows in plain fp32 torch, runs them through cdsl_gemv_noalloc in chunks of at most
-8 rows, and compares with the verify logits, for two rounds of calls in a row. This file is
-named so that pytest collects it last."""
+Some callers of this library cannot allocate device memory: host frameworks whose caching
+allocator already holds the GPU's memory, real-time loops that must not block on cudaMalloc,
+runtimes that forbid device allocation after start-up. cdsl_gemv_noalloc serves them: its
+scratch is a fixed array inside the library. The first test checks it against x @ w^T in fp64
+over every row count it takes (1..8), outputs that are not a multiple of the 128-row tile,
+inputs that are not a multiple of the 256-wide K step and the 8192 K limit, at 2e-5 of the
+sum of |x||w| (the hi/lo split of x keeps about 17 bits; the products and sums are fp32).
+The second builds a bf16 model whose layers leave the residual stream unchanged (the
+attention-output and FFN-down projections are zero), so cdsl_verify's logits are
+lm_head(RMSNorm(E[token])) for every verify row; it recomputes those normalized rows in fp32
+torch, runs them through cdsl_gemv_noalloc in chunks of at most 8 rows, and compares with the
+verify logits, for two rounds of calls in a row. This file is named so that pytest collects
+it last."""
 import numpy as np
 import pytest
 
@@ -19,6 +23,33 @@ from cdsl_parity import make_engine, make_setup
 pytestmark = pytest.mark.gpu
 
 TOL16 = 2e-2   # the bf16 logits tolerance of the parity tests
+REL = 2e-5     # of sum_k |x_k| |w_k|: the hi/lo split and fp32 accumulation
+
+
+@pytest.mark.parametrize("R,K,N", [(1, 768, 1000), (2, 1000, 129), (3, 2048, 3072),
+                                   (4, 8192, 4096), (5, 5504, 2048), (6, 1000, 32000),
+                                   (7, 8192, 1000), (8, 4096, 32000)])
+def test_noalloc_gemv_matches_fp64_product(R, K, N):
+    import torch
+    from paper_2412_10418_gb300 import build
+    build.build()
+    import paper_2412_10418_gb300 as cdsl
+
+    g = torch.Generator(device="cpu").manual_seed(1000 * R + K % 997)
+    w = (0.02 * torch.randn((N, K), generator=g)).to(torch.bfloat16).cuda()
+    x = torch.randn((R, K), generator=g).cuda()
+    ref = x.double() @ w.double().t()
+    bound = REL * (x.double().abs() @ w.double().abs().t()) + 1e-30
+    stream = torch.cuda.current_stream()
+    outs = []
+    for _ in range(2):                      # two calls in a row share the scratch
+        y = torch.full((R, N), float("nan"), dtype=torch.float32, device="cuda")
+        cdsl.cdsl_gemv_noalloc(w, x, y, stream.cuda_stream)
+        stream.synchronize()
+        excess = float(((y.double() - ref).abs() - bound).max())
+        assert excess <= 0.0, f"R={R} K={K} N={N}: error exceeds the bound by {excess:.3g}"
+        outs.append(y)
+    assert torch.equal(outs[0], outs[1])
 
 
 def test_noalloc_gemv_matches_verify_logits():
