@@ -51,6 +51,10 @@ def parse():
                          "7B-shape verify sweep instead of the step benchmark")
     ap.add_argument("--oracle-layers", type=int, default=2,
                     help="target layers the oracle sample runs (scaled to the full depth)")
+    ap.add_argument("--draft-equals-target", action="store_true",
+                    help="forced acceptance: the draft is the target model itself, so every "
+                         "lookahead is accepted and S1 steps emit several tokens")
+    ap.add_argument("--oracle-worker", default=None, help=argparse.SUPPRESS)
     return ap.parse_args()
 
 
@@ -73,12 +77,16 @@ def config_of(wl):
     }
 
 
+def streamed_weight_bytes_model(m):
+    """Weight bytes one forward pass of a bf16 model streams: every matrix but the embedding
+    table, whose rows are only gathered."""
+    return sum(math.prod(s) for n, s in m.weight_specs() if n != "embed") * 2
+
+
 def streamed_weight_bytes(wl):
     """Weight bytes one step reads through the projections: the target once, the draft once
-    per lookahead call (every matrix but the embedding table, whose rows are gathered)."""
-    def per_model(m):
-        return sum(math.prod(s) for n, s in m.weight_specs() if n != "embed") * 2
-    return per_model(wl.target) + wl.d * per_model(wl.draft)
+    per lookahead call."""
+    return streamed_weight_bytes_model(wl.target) + wl.d * streamed_weight_bytes_model(wl.draft)
 
 
 def gemm_traffic_ratio():
@@ -153,20 +161,26 @@ class ClockSampler:
 
 # ------------------------------------------------------------------------------ GPU arm
 
-def build_engine(wl, device, acceptance="hard", decoder="cdsl", step1_budget=0):
+def build_engine(wl, device, acceptance="hard", decoder="cdsl", step1_budget=0,
+                 draft_equals_target=False):
     """The CDSL-k engine of a workload. decoder "cdlh": M_p drafts its own lookaheads and the
     reward threshold is above any reward (S1 never holds), so every step emits the one token
     of Alg. 2's CDLH (the step still runs its verify pass, which scores the beams).
     "cdlh-appx": M_q's lookaheads, thresholds above any score: every step emits the one
-    CDLH-appx token c_{b*} (Alg. 2 with M_q as the lookahead model)."""
+    CDLH-appx token c_{b*} (Alg. 2 with M_q as the lookahead model).
+    draft_equals_target (CDSL only): M_p drafts its own lookaheads and r_t = 0, so every
+    lookahead is accepted and every step is S1, emitting c_b* and all d drafts (the forced
+    acceptance diagnostic of the S1 path: multi-token emission, multi-row KV commit, the
+    pending draft row of the next step)."""
     import torch
     import synth
     import paper_2412_10418_gb300 as cdsl
 
     tw = synth.model_weights(wl, "target", device=device)
-    cdlh = decoder == "cdlh"
+    cdlh = decoder == "cdlh" or draft_equals_target
     dw = tw if cdlh else synth.model_weights(wl, "draft", device=device)
     dshape = wl.target if cdlh else wl.draft
+    r_t = 0.0 if draft_equals_target else (2.0 if decoder != "cdsl" else wl.r_t)
     head = torch.from_numpy(synth.reward_head(wl)).to(device) if wl.reward_head else None
     eng = cdsl.Engine(wl.target, dshape, wl.dtype,
                       [tw[n] for n, _ in wl.target.weight_specs()],
@@ -174,7 +188,7 @@ def build_engine(wl, device, acceptance="hard", decoder="cdsl", step1_budget=0):
                       batch=wl.batch, k=wl.k, d=wl.d, max_prompt=wl.prompt_len,
                       max_new=wl.max_new, n_keywords=wl.n_keywords,
                       a_t=2.0 if decoder == "cdlh-appx" else wl.a_t,
-                      r_t=2.0 if decoder != "cdsl" else wl.r_t, reward_head=head,
+                      r_t=r_t, reward_head=head,
                       acceptance=cdsl.ACCEPT_SPECULATIVE if acceptance == "speculative"
                       else cdsl.ACCEPT_HARD, seed=1, step1_budget=step1_budget, device=device)
     return eng, tw, dw
@@ -223,26 +237,33 @@ def timed_steps(eng, wl, n_steps, warmup):
 
 
 def kernel_timing(eng, wl, n_steps):
-    """Per-launch CUDA events around every projection GEMM over n_steps steps (direct launches
-    on the engine's stream), and the verify call alone."""
+    """Kernel classes inside the graph-replayed step (cdsl_profile mode 2: the kernels stamp
+    their first block's entry and last block's exit; each launch is charged the part of its
+    interval after the previous stamped exit, so the charged times never add up to more than
+    the step), the same launches bracketed by CUDA events outside the graph (mode 1), and the
+    verify call alone between events."""
     import torch
     import paper_2412_10418_gb300 as cdsl
     prefill(eng, wl)
     eng.step()
-    cdsl.cdsl_profile(eng.ctx, True)
+
+    def read(mode):
+        prof = {name: cdsl.cdsl_get_profile(eng.ctx, impl)
+                for impl, name in cdsl.KERNEL_CLASSES.items()}
+        launches = cdsl.cdsl_get_profile_launches(eng.ctx)
+        if mode == cdsl.PROFILE_IN_GRAPH:
+            prof["_steps"] = cdsl.cdsl_get_profile(eng.ctx, cdsl.STAMPED_STEPS)
+        cdsl.cdsl_profile(eng.ctx, cdsl.PROFILE_OFF)
+        return prof, launches
+
+    cdsl.cdsl_profile(eng.ctx, cdsl.PROFILE_IN_GRAPH)
     for _ in range(n_steps):
         eng.step()
-    prof = {name: cdsl.cdsl_get_profile(eng.ctx, impl) for impl, name in cdsl.KERNEL_CLASSES.items()}
-    # tensor-core GEMM launches grouped by shape (equal algorithmic bytes = same projection)
-    groups = {}
-    for cls, ms, by, fl in cdsl.cdsl_get_profile_launches(eng.ctx):
-        if cls != 2:
-            continue
-        g = groups.setdefault(round(by), [0, 0.0])
-        g[0] += 1
-        g[1] += ms
-    cdsl.cdsl_profile(eng.ctx, False)
-    prof["_gemm_shapes"] = groups
+    in_graph = read(cdsl.PROFILE_IN_GRAPH)
+    cdsl.cdsl_profile(eng.ctx, cdsl.PROFILE_EVENTS)
+    for _ in range(n_steps):
+        eng.step()
+    events = read(cdsl.PROFILE_EVENTS)
     # verify-step time: lookahead, then the verify call alone between events
     ts = []
     for _ in range(n_steps):
@@ -254,7 +275,30 @@ def kernel_timing(eng, wl, n_steps):
         eng.select()
         eng.stream.synchronize()
         ts.append(e0.elapsed_time(e1))
-    return prof, statistics.median(ts) * 1000.0
+    return in_graph, events, statistics.median(ts) * 1000.0
+
+
+def by_shape(launches, cls, per_step_div, hbm):
+    """Launches of one class grouped by algorithmic bytes (one group per projection shape),
+    largest total time first. In mode 2 a launch record's milliseconds are already per step;
+    in mode 1 they are per launch (per_step_div = steps profiled)."""
+    groups = {}
+    for c, ms, by, fl in launches:
+        if c != cls or by <= 0:
+            continue
+        g = groups.setdefault(round(by), [0, 0.0])
+        g[0] += 1
+        g[1] += ms
+    rows = []
+    for b, (n, ms) in groups.items():
+        if ms <= 0:
+            continue
+        per_launch_ms = ms / n
+        gbs = b / (per_launch_ms / 1000.0) / 1e9
+        rows.append({"bytes_per_launch": b, "launches_per_step": round(n / per_step_div, 2),
+                     "avg_us": round(per_launch_ms * 1000.0, 2), "GB/s": round(gbs, 1),
+                     "frac": round(gbs / hbm, 3)})
+    return sorted(rows, key=lambda r: -r["avg_us"] * r["launches_per_step"])
 
 
 def e2e_run(eng, wl, n_steps):
@@ -298,71 +342,131 @@ def e2e_run(eng, wl, n_steps):
 
 # ------------------------------------------------------------------------------ oracle arm
 
-def oracle_sample(wl, tw_host_fn, dw_host, n_layers, steps=1, warmup=0):
-    """The oracle as it stands on a bounded sample of the workload: CDSL-k steps of the
-    7B-shaped models over a 16-token prompt with the target cut to its first n_layers layers.
-    Returns (seconds per full step, scaled to the full target depth, cores)."""
+ORACLE_PREFIX = "oracle_"
+
+
+def cut_shape(shape, n_layers):
+    import synth
+    return synth.ModelShape(n_layers=n_layers, d_model=shape.d_model, n_heads=shape.n_heads,
+                            n_kv_heads=shape.n_kv_heads, d_ffn=shape.d_ffn, vocab=shape.vocab,
+                            rope_theta=shape.rope_theta, norm_eps=shape.norm_eps)
+
+
+def oracle_worker(args):
+    """The oracle as it stands, in a process of its own (its BLAS thread count is fixed by the
+    environment the parent gives it): CDSL-k steps of the first prompt of the workload on its
+    real prompt, the draft at full depth and the target cut to its first --oracle-layers
+    layers (plus embedding, final norm and LM head). The first worker prefills and saves the
+    decoding state; later workers start from that saved state. Prints one JSON line."""
+    import pickle
     import numpy as np
     import synth
     import oracle
-    tshape = wl.target
-    cut = synth.ModelShape(n_layers=n_layers, d_model=tshape.d_model, n_heads=tshape.n_heads,
-                           n_kv_heads=tshape.n_kv_heads, d_ffn=tshape.d_ffn, vocab=tshape.vocab)
-    tgt = oracle.Transformer(cut, tw_host_fn(n_layers), keep_widened=False)
-    drf = oracle.Transformer(wl.draft, dw_host, keep_widened=True)
-    for name in dw_host:          # the draft's fp64 copies are cached by the oracle after use
-        drf.w(name)
+    wdir = args.oracle_worker
+    meta = json.load(open(os.path.join(wdir, "meta.json")))
+    wl = synth.WORKLOADS[meta["workload"]]
+    n_cut = meta["layers"]
+    def load(prefix):
+        return {f[len(prefix):-4]: np.load(os.path.join(wdir, f), mmap_mode="r")
+                for f in os.listdir(wdir) if f.startswith(prefix) and f.endswith(".npy")}
+    tgt = oracle.Transformer(cut_shape(wl.target, n_cut), load("t_"), keep_widened=True)
+    drf = oracle.Transformer(wl.draft, load("d_"), keep_widened=True)
+    for m in (tgt, drf):                  # widen every matrix once, before any timing
+        for name in m.raw:
+            m.w(name)
     run = oracle.RunParams(k=wl.k, d=wl.d, a_t=wl.a_t, r_t=wl.r_t, max_new=10_000,
                            composite_reward=wl.reward_head)
-    prompt = synth.prompts(wl)[:1, :16]
-    states = oracle.prefill(tgt, drf, prompt, synth.keywords(wl)[:1])
-    w = synth.reward_head(wl)
-    for _ in range(warmup):
-        oracle.cdsl_k_step(tgt, drf, states, run, w)
-    t_draft = t_tgt = 0.0
-    for _ in range(steps):
-        # the same step split into its two model parts, to scale the target part
+    w_head = synth.reward_head(wl)
+    st_path = os.path.join(wdir, "states.pkl")
+    prefill_s = None
+    if os.path.exists(st_path):
+        states = pickle.load(open(st_path, "rb"))
+    else:
         t0 = time.perf_counter()
-        dcs = [states[0].dcache.fork() for _ in range(wl.k)]
-        roots = np.argsort(-states[0].p_root)[:wl.k].tolist()
-        feed = roots
-        xs = [[] for _ in range(wl.k)]
-        for j in range(wl.d):
-            lg, _ = drf.forward([(dcs[i], [feed[i]]) for i in range(wl.k)])
-            feed = [int(np.argmax(l[0])) for l in lg]
-            for i in range(wl.k):
-                xs[i].append(feed[i])
+        states = oracle.prefill(tgt, drf, synth.prompts(wl)[:1], synth.keywords(wl)[:1])
+        prefill_s = time.perf_counter() - t0
+        pickle.dump(states, open(st_path, "wb"))
+    step_s, tgt_s, tokens = [], [], 0
+    for i in range(meta["warmup"] + meta["steps"]):
+        t0 = time.perf_counter()
+        rec = oracle.cdsl_k_step(tgt, drf, states, run, w_head)[0]
         t1 = time.perf_counter()
-        tgt.forward([(states[0].tcache.fork(), [roots[i]] + xs[i]) for i in range(wl.k)])
+        # the step's target pass alone (same rows, a forked cache), for the depth scaling
+        tgt.forward([(states[0].tcache.fork(), [int(rec.roots[j])] + rec.x[j].tolist())
+                     for j in range(wl.k)])
         t2 = time.perf_counter()
-        t_draft += t1 - t0
-        t_tgt += t2 - t1
-    per_layer = t_tgt / steps / n_layers
-    step_s = t_draft / steps + per_layer * tshape.n_layers
-    return step_s, os.cpu_count()
+        if i >= meta["warmup"]:
+            step_s.append(t1 - t0)
+            tgt_s.append(t2 - t1)
+            tokens += len(rec.emitted)
+    print(json.dumps({"threads": int(os.environ.get("OPENBLAS_NUM_THREADS", "0") or 0),
+                      "prefill_s": prefill_s, "step_s": step_s, "target_s": tgt_s,
+                      "tokens": tokens}), flush=True)
 
 
-def host_weights_fns(wl, tw, dw):
+def oracle_runs(wl, tw, dw, n_layers, runs):
+    """Run oracle_worker processes on the host cores: runs = [(threads, warmup, steps), ...],
+    the first of them also prefilling the real prompt. tw / dw: the engine's weights (torch
+    tensors, any device). Returns one result dict per run, with the depth-scaled estimate of
+    a full-depth step added (the target's share scaled by the streamed weights of the full
+    target over those of the cut one: the verify pass's flops are proportional to them)."""
+    import shutil
+    import numpy as np
     import synth
+    keep_t = {"embed", "final_norm", "lm_head"} | {
+        f"l{l}.{x}" for l in range(n_layers)
+        for x in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down")}
+    wdir = tempfile.mkdtemp(prefix="cdsl_oracle_")
+    try:
+        for prefix, src, keep in (("t_", tw, keep_t), ("d_", dw, None)):
+            for name, arr in synth.to_host({k: v for k, v in src.items()
+                                            if keep is None or k in keep}).items():
+                np.save(os.path.join(wdir, prefix + name + ".npy"), arr)
+        out = []
+        for threads, warmup, steps in runs:
+            json.dump({"workload": wl.name, "layers": n_layers, "warmup": warmup,
+                       "steps": steps}, open(os.path.join(wdir, "meta.json"), "w"))
+            env = dict(os.environ, OPENBLAS_NUM_THREADS=str(threads), OMP_NUM_THREADS=str(threads),
+                       MKL_NUM_THREADS=str(threads))
+            r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-worker", wdir],
+                               env=env, capture_output=True, text=True, timeout=1800)
+            if r.returncode != 0:
+                raise RuntimeError(f"oracle worker ({threads} threads) failed: {r.stderr[-2000:]}")
+            res = json.loads(r.stdout.strip().splitlines()[-1])
+            ratio = (streamed_weight_bytes_model(wl.target) /
+                     streamed_weight_bytes_model(cut_shape(wl.target, n_layers)))
+            n = max(1, len(res["step_s"]))
+            res["sample_step_s"] = sum(res["step_s"]) / n
+            res["full_depth_step_s"] = (sum(res["step_s"]) + (ratio - 1.0) * sum(res["target_s"])) / n
+            res["tokens_per_step"] = res["tokens"] / n
+            out.append(res)
+        return out
+    finally:
+        shutil.rmtree(wdir, ignore_errors=True)
 
-    def target_cut(n):
-        keep = {"embed", "final_norm", "lm_head"} | {f"l{l}.{x}" for l in range(n) for x in
-                                                      ("attn_norm", "wq", "wk", "wv", "wo",
-                                                       "ffn_norm", "w_gate", "w_up", "w_down")}
-        return synth.to_host({k: v for k, v in tw.items() if k in keep})
 
-    return target_cut, synth.to_host(dw)
+def oracle_sample_text(wl, n_layers):
+    return (f"CDSL-k steps of the fp64 oracle on the workload's first prompt ({wl.prompt_len} "
+            f"tokens, prefilled once), k={wl.k}, d={wl.d}: the draft at its full "
+            f"{wl.draft.n_layers} layers, the target cut to {n_layers} of "
+            f"{wl.target.n_layers} layers; the measured step is scaled to the full target depth "
+            "by the ratio of streamed target weights (the verify pass's flops follow them)")
 
 
-def cpu_baseline(wl, tw, dw, tokens_per_step, n_layers):
-    fn, dh = host_weights_fns(wl, tw, dw)
-    step_s, cores = oracle_sample(wl, fn, dh, n_layers)
-    return {"value": tokens_per_step * wl.batch / step_s, "unit": "tokens/s", "cores": cores,
-            "kind": "oracle",
-            "sample": (f"one CDSL-k step (B=1, k={wl.k}, d={wl.d}) of the fp64 oracle on a "
-                       f"16-token prompt: draft {wl.d} calls x {wl.k} beams in full, target "
-                       f"{n_layers} of {wl.target.n_layers} layers timed and scaled to the full "
-                       f"depth; {tokens_per_step:.2f} tokens/step as measured on the GPU")}
+def cpu_baseline(wl, tw, dw, n_layers):
+    """The oracle timed on the host cores at all cores and at 1 thread, one step each after
+    the prefill (value: all cores, full-depth estimate)."""
+    cores = os.cpu_count()
+    allc, one = oracle_runs(wl, tw, dw, n_layers, [(cores, 0, 1), (1, 0, 1)])
+    def summary(r):
+        return {"threads": r["threads"], "sample_ms_per_step": round(r["sample_step_s"] * 1e3, 1),
+                "full_depth_ms_per_step_estimate": round(r["full_depth_step_s"] * 1e3, 1),
+                "tokens_per_s": round(r["tokens_per_step"] / r["full_depth_step_s"], 6)}
+    return {"value": round(allc["tokens_per_step"] / allc["full_depth_step_s"], 6),
+            "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": oracle_sample_text(wl, n_layers),
+            "prefill_s": round(allc["prefill_s"], 1) if allc["prefill_s"] else None,
+            "all_cores": summary(allc), "one_thread": summary(one)}
 
 
 # ------------------------------------------------------------------------------ ranks
@@ -408,7 +512,8 @@ def gpu_main(args):
     if world > 1:
         dist.barrier()
     wl = workload(args.workload)
-    eng, tw, dw = build_engine(wl, device, args.acceptance, args.decoder, args.step1_budget)
+    eng, tw, dw = build_engine(wl, device, args.acceptance, args.decoder, args.step1_budget,
+                               args.draft_equals_target)
 
     if world > 1:
         dist.barrier()
@@ -422,39 +527,62 @@ def gpu_main(args):
     launches_per_step = counters[6]
 
     n_prof = min(args.steps, 5)
-    prof, verify_us = kernel_timing(eng, wl, n_prof)
-    shapes = prof.pop("_gemm_shapes")
+    (prof, launches), (prof_ev, launches_ev), verify_us = kernel_timing(eng, wl, n_prof)
     import paper_2412_10418_gb300 as cdsl
-    gem = {k: v for k, v in prof.items() if k in cdsl.GEMM_IMPLS.values()}
-    dom = max(gem.items(), key=lambda kv: kv[1]["ms"])
     pk = peaks()
     hbm = pk["hbm_gbs"] if pk else 6800.0
-    achieved = dom[1]["bytes"] / (dom[1]["ms"] / 1000.0) / 1e9 if dom[1]["ms"] > 0 else 0.0
+    step_ms = total_ms / args.steps   # every rank times args.steps steps; the slowest rank
+    stamped = prof.pop("_steps")
+    gem = {k: v for k, v in prof.items() if k in cdsl.GEMM_IMPLS.values()}
+    dom = max(gem.items(), key=lambda kv: kv[1]["ms"])
+    d = dom[1]
+    n_launch = max(1, d["launches"])
+    avg_ms = d["ms"] / n_launch
+    bpl = d["bytes"] / n_launch
+    achieved = bpl / (avg_ms / 1000.0) / 1e9 if avg_ms > 0 else 0.0
     ratio = gemm_traffic_ratio() if dom[0] == "gemm_tc" else None
-    bpl = dom[1]["bytes"] / max(1, dom[1]["launches"])
+    charged = sum(v["ms"] for v in prof.values()) / n_prof
     roofline = {"bound": "hbm", "kernel": dom[0], "achieved": round(achieved, 1),
                 "peak": hbm, "unit": "GB/s", "frac": round(achieved / hbm, 4),
                 "traffic": round(ratio * bpl) if ratio else None,
                 "peak_source": "measured" if pk else "fallback",
-                "timing": "CUDA events around each launch, direct launches (no graph overlap)",
-                "launches_timed": dom[1]["launches"],
-                "avg_launch_us": round(dom[1]["ms"] * 1000.0 / max(1, dom[1]["launches"]), 2),
-                "bytes_per_launch": round(dom[1]["bytes"] / max(1, dom[1]["launches"]))}
-    # per projection shape (the same kernel, different launch shapes): the largest by time
-    by_shape = sorted(({"bytes_per_launch": b, "launches": n, "avg_us": round(ms * 1000.0 / n, 2),
-                        "GB/s": round(b / (ms / n / 1000.0) / 1e9, 1),
-                        "frac": round(b / (ms / n / 1000.0) / 1e9 / hbm, 3)}
-                       for b, (n, ms) in shapes.items()), key=lambda r: -r["avg_us"] * r["launches"])
-    roofline["by_shape"] = by_shape[:8]
-    # the same bytes over the graph-replayed step (everything else in the step included): a
-    # lower bound on the projections' rate inside the CUDA graph
-    step_bytes = dom[1]["bytes"] / n_prof
-    step_ms = total_ms / args.steps   # every rank times args.steps steps; the slowest rank
-    roofline["in_graph_lower_bound"] = {
-        "bytes_per_step": round(step_bytes), "ms_per_step": round(step_ms, 4),
-        "GB/s": round(step_bytes / (step_ms / 1000.0) / 1e9, 1),
-        "frac": round(step_bytes / (step_ms / 1000.0) / 1e9 / hbm, 4)}
-    verify_bytes = (wl.target.n_params() * 2)
+                "timing": "in the CUDA graph: per-launch %globaltimer stamps (first block "
+                          "entry, last block exit), each launch charged after the previous "
+                          "stamped exit; the charged times of a step never overlap",
+                "launches_per_step": round(d["launches"] / n_prof, 1),
+                "avg_launch_us": round(avg_ms * 1000.0, 2),
+                "bytes_per_launch": round(bpl),
+                "ms_per_step_in_graph": round(d["ms"] / n_prof, 4),
+                "stamped_step_ms": round(stamped["ms"] / max(1, stamped["launches"]), 4),
+                "charged_ms_per_step_all_classes": round(charged, 4)}
+    roofline["by_shape"] = by_shape(launches, 2, 1, hbm)[:10]
+    att = prof.get("attention", {})
+    if att.get("ms"):
+        a_bpl = att["bytes"] / max(1, att["launches"])
+        a_ms = att["ms"] / max(1, att["launches"])
+        a_gbs = a_bpl / (a_ms / 1000.0) / 1e9
+        roofline["attention"] = {
+            "bound": "hbm", "launches_per_step": round(att["launches"] / n_prof, 1),
+            "avg_launch_us": round(a_ms * 1000.0, 2), "bytes_per_launch": round(a_bpl),
+            "achieved": round(a_gbs, 1), "frac": round(a_gbs / hbm, 4),
+            "ms_per_step_in_graph": round(att["ms"] / n_prof, 4),
+            "bytes": "counted by the kernel: K and V (fp32) of every key once per prompt and "
+                     "KV head, every query vector read and its output written once"}
+    roofline["in_graph_ms_per_step"] = {k: round(v["ms"] / n_prof, 4) for k, v in prof.items()
+                                        if v["ms"] > 0}
+    # the same launches bracketed by CUDA events outside the graph (no overlap between them)
+    dev = prof_ev.get(dom[0], {})
+    if dev.get("ms"):
+        ev_ms = dev["ms"] / max(1, dev["launches"])
+        ev_bpl = dev["bytes"] / max(1, dev["launches"])
+        roofline["event_timed"] = {
+            "timing": "CUDA events around each launch on the engine's stream, direct launches "
+                      "(no graph, no programmatic overlap)",
+            "avg_launch_us": round(ev_ms * 1000.0, 2),
+            "achieved": round(ev_bpl / (ev_ms / 1000.0) / 1e9, 1),
+            "frac": round(ev_bpl / (ev_ms / 1000.0) / 1e9 / hbm, 4),
+            "by_shape": by_shape(launches_ev, 2, n_prof, hbm)[:10]}
+    verify_bytes = streamed_weight_bytes_model(wl.target)
     e2e = None
     if not args.no_e2e:
         ev, h2d, d2h, n_e2e = e2e_run(eng, wl, args.steps)
@@ -469,8 +597,9 @@ def gpu_main(args):
     if rank == 0:
         tokens_per_step = tokens / (args.steps * max(1, world)) / wl.batch
         cpu = None
-        if not args.no_cpu_baseline and world == 1 and args.decoder == "cdsl":
-            cpu = cpu_baseline(wl, tw, dw, tokens_per_step, args.oracle_layers)
+        if (not args.no_cpu_baseline and world == 1 and args.decoder == "cdsl"
+                and not args.draft_equals_target):
+            cpu = cpu_baseline(wl, tw, dw, args.oracle_layers)
         out = {
             "metric": METRIC, "value": round(value, 3), "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
@@ -481,14 +610,18 @@ def gpu_main(args):
                            step1_budget=args.step1_budget,
                            **({"draft": "= target (CDLH)", "r_t": None}
                               if args.decoder == "cdlh" else {}),
-                           **({"a_t": None, "r_t": None} if args.decoder == "cdlh-appx" else {})),
+                           **({"a_t": None, "r_t": None} if args.decoder == "cdlh-appx" else {}),
+                           **({"draft": "= target (forced acceptance)", "r_t": 0.0}
+                              if args.draft_equals_target else {})),
             "verify_us": round(verify_us, 1),
             "verify_gbs": round(verify_bytes / (verify_us * 1e-6) / 1e9, 1),
             "tokens_per_step": round(tokens_per_step, 3),
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
             "gpu_launches": int(launches_per_step * args.steps),
-            "kernel_profile": {k: {"launches": v["launches"], "ms_per_step": round(v["ms"] / n_prof, 3),
-                                   "GB/s": round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1) if v["bytes"] else None}
+            "kernel_profile": {k: {"launches_per_step": round(v["launches"] / n_prof, 1),
+                                   "ms_per_step_in_graph": round(v["ms"] / n_prof, 4),
+                                   "GB/s": (round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1)
+                                            if v["bytes"] and v["ms"] else None)}
                                for k, v in prof.items() if v["launches"]},
         }
         print(json.dumps(out), flush=True)
@@ -499,8 +632,9 @@ def gpu_main(args):
 
 
 def reference_main(args):
-    """The oracle arm: the fp64 oracle as it stands on the host cores, each step a bounded
-    sample of the same workload (rank 0 only; other ranks exit without work)."""
+    """The oracle arm: the fp64 oracle as it stands on the host cores (all of them), each step
+    a bounded sample of the same workload (see oracle_sample_text); one more step at one
+    thread for the single-core figure. Rank 0 only; other ranks exit without work."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
@@ -508,25 +642,34 @@ def reference_main(args):
     wl = workload(args.workload)
     device = "cuda:0" if torch.cuda.is_available() else "cpu"
     import synth
-    # weights drawn exactly as the GPU arm draws them, then copied to the host
+    # weights drawn exactly as the GPU arm draws them (7B/13B shapes on the GPU)
     tw = synth.model_weights(wl, "target", device=device)
     dw = synth.model_weights(wl, "draft", device=device)
-    fn, dh = host_weights_fns(wl, tw, dw)
-    del tw, dw
-    step_s, cores = oracle_sample(wl, fn, dh, args.oracle_layers, steps=args.steps,
-                                  warmup=args.warmup)
-    value = wl.batch / step_s   # one token per prompt and step (the GPU arm's measured rate)
-    sample = (f"per step: one CDSL-k step (B=1, k={wl.k}, d={wl.d}) of the fp64 oracle on a "
-              f"16-token prompt, target {args.oracle_layers} of {wl.target.n_layers} layers "
-              "timed and scaled to the full depth; 1 token per step")
+    cores = os.cpu_count()
+    t_start = time.perf_counter()
+    allc, one = oracle_runs(wl, tw, dw, args.oracle_layers,
+                            [(cores, args.warmup, args.steps), (1, 0, 1)])
+    wall = time.perf_counter() - t_start
+    value = allc["tokens_per_step"] / allc["full_depth_step_s"]
+    summ = lambda r: {"threads": r["threads"],
+                      "sample_ms_per_step": round(r["sample_step_s"] * 1e3, 1),
+                      "full_depth_ms_per_step_estimate": round(r["full_depth_step_s"] * 1e3, 1),
+                      "tokens_per_s": round(r["tokens_per_step"] / r["full_depth_step_s"], 6)}
     out = {"metric": METRIC, "value": round(value, 6), "unit": "tokens/s", "n_gpus": 1,
-           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(step_s * 1e3, 1),
+           "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": round(allc["sample_step_s"] * 1e3, 1),
+           "ms_per_step_note": "measured: one sample step (the cut target); value uses the "
+                               "full-depth estimate",
+           "ms_per_step_full_depth_estimate": round(allc["full_depth_step_s"] * 1e3, 1),
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "impl": "reference", "config": config_of(wl),
            "cpu_baseline": {"value": round(value, 6), "unit": "tokens/s", "kind": "oracle",
-                            "cores": cores, "sample": sample},
+                            "cores": cores, "sample": oracle_sample_text(wl, args.oracle_layers),
+                            "prefill_s": round(allc["prefill_s"], 1) if allc["prefill_s"] else None,
+                            "all_cores": summ(allc), "one_thread": summ(one)},
            "e2e": {"value": round(value, 6), "unit": "tokens/s", "h2d_bytes_per_step": 0,
-                   "d2h_bytes_per_step": 0}}
+                   "d2h_bytes_per_step": 0},
+           "wall_s": round(wall, 1)}
     print(json.dumps(out), flush=True)
 
 
@@ -545,7 +688,7 @@ def verify_sweep(args):
     tw = synth.model_weights(wl0, "target", device="cuda")
     dw = synth.model_weights(wl0, "draft", device="cuda")
     head = torch.from_numpy(synth.reward_head(wl0)).cuda()
-    wbytes = wl0.target.n_params() * 2
+    wbytes = streamed_weight_bytes_model(wl0.target)
     pk = peaks()
     hbm = pk["hbm_gbs"] if pk else 6800.0
     tfl = pk.get("bf16_tflops") if pk else None
@@ -594,7 +737,9 @@ def verify_sweep(args):
 
 if __name__ == "__main__":
     a = parse()
-    if a.impl == "reference":
+    if a.oracle_worker:
+        oracle_worker(a)
+    elif a.impl == "reference":
         reference_main(a)
     elif a.verify_sweep:
         verify_sweep(a)

@@ -194,22 +194,34 @@ CDSL_API int32_t cdsl_get_tokens(cdsl_ctx* ctx, int32_t* d_tokens, int32_t* d_le
  * call. */
 CDSL_API int32_t cdsl_get_counters(cdsl_ctx* ctx, int64_t* h_counters);
 
-/* Kernel timing (a measurement aid; the paper has no counterpart). With enable != 0 every
- * kernel launch of the following calls is bracketed by CUDA events on the context's stream
- * and cdsl_step launches its kernels directly instead of through its graph.
+/* Kernel timing (a measurement aid; the paper has no counterpart). cdsl_profile(ctx, mode):
+ *   0: off.
+ *   1: every kernel launch of the following calls is bracketed by CUDA events on the
+ *      context's stream, and cdsl_step launches its kernels directly instead of through its
+ *      graph (per-launch durations without the overlap of programmatic dependent launch).
+ *   2: in-graph timing. cdsl_step replays a second graph whose GEMM, attention and row
+ *      statistics kernels stamp their first block's entry and last block's exit on the device
+ *      clock (%globaltimer); after each step the call synchronizes the stream and charges
+ *      every stamped launch, in stream order, from its entry (or the previous stamped exit,
+ *      whichever is later) to its exit. The charged intervals are disjoint, so their sum
+ *      never exceeds the step. The attention kernel also counts its own algorithmic bytes
+ *      (K and V of every key once per prompt and KV head, queries and outputs once).
  * cdsl_get_profile synchronizes the stream and returns, for kernel class `impl`
  * (0 = CUDA-core tiled GEMM, 1 = weight-streaming GEMV, 2 = tcgen05 tensor-core GEMM,
  * 3 = attention, 4 = RMSNorm, 5 = logits row statistics, 6 = embedding, 7 = plans, decision
- * and commit; bytes and flops are filled in for the GEMM classes only),
+ * and commit; in mode 2 also 8 = the stamped steps: {steps, milliseconds from the first
+ * stamped entry to the last stamped exit, 0, 0}),
  * h_out[4] = {launches, total milliseconds, algorithmic bytes (weights read once, activations
- * read, outputs written), flops} over the launches recorded since cdsl_profile last enabled
- * or disabled timing (each call of cdsl_profile clears the record). */
+ * read, outputs written; attention as counted by the kernel), flops} over the launches
+ * recorded since cdsl_profile was last called (each call clears the record). In mode 2 the
+ * classes 4, 6 and 7 are not stamped and report 0 milliseconds. */
 CDSL_API int32_t cdsl_profile(cdsl_ctx* ctx, int32_t enable);
 CDSL_API int32_t cdsl_get_profile(cdsl_ctx* ctx, int32_t impl, double* h_out);
 /* Per-launch form of the same record: for each of the first h_capacity recorded launches,
  * in launch order, four doubles {class, milliseconds, algorithmic bytes, flops} at h_out
- * [4 * i]; returns the number of records written (>= 0) or a negative status. Synchronizes
- * the stream. */
+ * [4 * i] (mode 2: one record per launch of the stamped step, milliseconds and bytes
+ * averaged over the stamped steps); returns the number of records written (>= 0) or a
+ * negative status. Synchronizes the stream. */
 CDSL_API int32_t cdsl_get_profile_launches(cdsl_ctx* ctx, double* h_out, int32_t h_capacity);
 
 /* Step-1 round 2 of the last cdsl_select / cdsl_step (budget 2; Alg. 1, S2/S3 Step-1): d_need [B]

@@ -193,13 +193,19 @@ def cdsl_get_status(ctx) -> int:
     return v.value
 
 
-def cdsl_profile(ctx, enable: bool):
-    _check(lib().cdsl_profile(ctx, int(bool(enable))), ctx)
+PROFILE_OFF, PROFILE_EVENTS, PROFILE_IN_GRAPH = 0, 1, 2
+
+
+def cdsl_profile(ctx, mode):
+    """mode 0 off, 1 CUDA events around direct launches, 2 in-graph stamps (see cdsl.h);
+    True / False stand for 1 / 0."""
+    _check(lib().cdsl_profile(ctx, int(mode)), ctx)
 
 
 GEMM_IMPLS = {0: "gemm_simt", 1: "gemv_stream", 2: "gemm_tc"}
 KERNEL_CLASSES = {0: "gemm_simt", 1: "gemv_stream", 2: "gemm_tc", 3: "attention", 4: "rmsnorm",
                   5: "row_stats", 6: "embed", 7: "step_logic"}
+STAMPED_STEPS = 8   # cdsl_get_profile class of the stamped steps themselves (mode 2)
 
 
 def cdsl_get_profile(ctx, impl: int):

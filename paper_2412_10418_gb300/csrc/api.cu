@@ -85,9 +85,21 @@ struct cdsl_ctx {
   int phase = PH_NEW;
   cudaGraphExec_t graph = nullptr;
   long long graph_nodes = 0;
-  // kernel timing (cdsl_profile)
+  // kernel timing (cdsl_profile): mode 1 events around direct launches, mode 2 in-graph stamps
   struct ProfRec { int impl; double bytes, flops; size_t ev; };
-  bool profiling = false;
+  int prof_mode = 0;
+  bool profiling = false;       // mode 1
+  // mode 2: launch records of the stamped graph (LaunchStamp; kStampStride apart)
+  unsigned long long* stamps = nullptr;   // [3][kStampStride]
+  bool stamping = false;        // capturing the stamped graph
+  unsigned long long* cur_stamp = nullptr;   // record of the launch being issued
+  cudaGraphExec_t graph_st = nullptr;
+  struct StampRec { int impl; double bytes, flops; };
+  std::vector<StampRec> st_recs;          // per launch of the stamped step, in stream order
+  std::vector<double> st_ms;              // attributed in-graph milliseconds per launch, summed
+  std::vector<double> st_kbytes;          // kernel-counted bytes per launch, summed
+  int st_steps = 0;
+  double st_span_ms = 0;                  // first stamped entry to last stamped exit, summed
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   std::vector<ProfRec> prof;
@@ -330,6 +342,7 @@ size_t carve(cdsl_ctx* c, void* base) {
   s.s1_reward = cv.take<float>(B);
   s.s1_topk = cv.take<int32_t>((size_t)B * k);
   s.s1_used = cv.take<int32_t>(B);
+  c->stamps = cv.take<unsigned long long>((size_t)3 * kStampStride);
   return (cv.off + 255) & ~size_t(255);
 }
 
@@ -359,6 +372,14 @@ enum { K_GEMM_SIMT = 0, K_GEMV = 1, K_GEMM_TC = 2, K_ATTN = 3, K_NORM = 4, K_ROW
 
 template <typename F>
 void timed(cdsl_ctx* c, int cls, double bytes, double flops, F&& launch) {
+  if (c->stamping) {   // capturing the stamped graph: give the launch its record
+    const size_t i = c->st_recs.size();
+    c->cur_stamp = i < (size_t)kStampStride ? c->stamps + i : nullptr;
+    c->st_recs.push_back({cls, bytes, flops});
+    launch();
+    c->cur_stamp = nullptr;
+    return;
+  }
   if (!c->profiling) {
     launch();
     return;
@@ -383,10 +404,12 @@ void gemm(cdsl_ctx* c, const GemmArgs& a) {
   const bool bf16 = c->dtype == CDSL_DTYPE_BF16;
   const int impl = (bf16 && tc_supported(a)) ? K_GEMM_TC : (bf16 && a.R <= 8) ? K_GEMV : K_GEMM_SIMT;
   double fl = 0;
-  const double by = c->profiling ? gemm_bytes(c, a, &fl) : 0.0;
+  const double by = (c->profiling || c->stamping) ? gemm_bytes(c, a, &fl) : 0.0;
+  GemmArgs as = a;   // as launched: with the launch's timing record, if any
   if (impl == K_GEMV) {
     timed(c, impl, by, fl, [&] {
-      launch_gemv(a, plan_gemv(a.K, a.n_virtual, kPlanSMs), c->gemv_part, c->gemv_cnt, c->stream);
+      as.stamp = c->cur_stamp;
+      launch_gemv(as, plan_gemv(a.K, a.n_virtual, kPlanSMs), c->gemv_part, c->gemv_cnt, c->stream);
     });
   } else if (impl == K_GEMM_TC) {
     TcMaps maps;
@@ -399,9 +422,15 @@ void gemm(cdsl_ctx* c, const GemmArgs& a) {
     // activation boxes: 64 features x n_pad rows (<= 256 <= R_pad), one per plane and stage
     maps.xh = tensor_map(c, xb, a.ldx, c->R_pad, p.n_pad);
     maps.xl = tensor_map(c, xb + a.x_plane, a.ldx, c->R_pad, p.n_pad);
-    timed(c, impl, by, fl, [&] { launch_gemm_tc(maps, a, p, c->gemv_part, c->gemv_cnt, c->stream); });
+    timed(c, impl, by, fl, [&] {
+      as.stamp = c->cur_stamp;
+      launch_gemm_tc(maps, as, p, c->gemv_part, c->gemv_cnt, c->stream);
+    });
   } else {
-    timed(c, impl, by, fl, [&] { launch_gemm_simt(c->dtype, a, c->stream); });
+    timed(c, impl, by, fl, [&] {
+      as.stamp = c->cur_stamp;
+      launch_gemm_simt(c->dtype, as, c->stream);
+    });
   }
 }
 
@@ -497,7 +526,11 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     normed_input(q, c->ss_a);
     gemm(c, q);
     at.layer = l;
-    timed(c, K_ATTN, 0, 0, [&] { launch_attn(c->dtype, at, n_z, s); });
+    timed(c, K_ATTN, 0, 0, [&] {
+      at.stamp = c->cur_stamp;
+      launch_attn(c->dtype, at, n_z, s);
+      at.stamp = nullptr;
+    });
     GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->Xa, H * hd, R);
     o.w[0] = W[W_O]; o.seg_rows[0] = D; o.n_seg = 1; o.n_virtual = D;
     residual_out(o, W[W_FFN_NORM], c->ss_b, false);
@@ -544,7 +577,10 @@ void do_lookahead(cdsl_ctx* c) {
     a.logits = c->logits; a.R = c->B * c->k; a.V = c->V; a.k = c->k;
     a.x_out = c->st.x; a.logq_out = c->st.logq; a.out_stride = c->d; a.out_off = j - 1;
     a.status = c->st.status;
-    timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
+    timed(c, K_ROWSTATS, 0, 0, [&] {
+      a.stamp = c->cur_stamp;
+      launch_row_stats(a, c->stream);
+    });
   }
 }
 
@@ -562,7 +598,10 @@ void do_verify(cdsl_ctx* c) {
     a.ss = c->ss_a; a.hw = c->ss_hw; a.norm_D = c->tcfg.d_model; a.ld_ss = c->R_pad;
     a.norm_eps = c->tcfg.norm_eps; a.head_out = c->st.v_head;
   }
-  timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
+  timed(c, K_ROWSTATS, 0, 0, [&] {
+      a.stamp = c->cur_stamp;
+      launch_row_stats(a, c->stream);
+    });
 }
 
 // Step-1 round 2 (Alg. 1 S2/S3, budget b = 2) for every prompt: d draft calls from
@@ -581,7 +620,10 @@ void do_step1_round(cdsl_ctx* c) {
     a.logits = c->logits; a.R = B; a.V = c->V; a.k = c->k;
     a.x_out = c->st.s1_tok; a.logq_out = c->st.s1_logq; a.out_stride = d + 1; a.out_off = j;
     a.status = c->st.status;
-    timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
+    timed(c, K_ROWSTATS, 0, 0, [&] {
+      a.stamp = c->cur_stamp;
+      launch_row_stats(a, c->stream);
+    });
   }
   timed(c, K_STEPLOGIC, 0, 0, [&] { launch_plan_s1_verify(c->st, c->rows_v, c->stream); });
   AttnPass ap;
@@ -591,7 +633,10 @@ void do_step1_round(cdsl_ctx* c) {
   RowStatsArgs a{};
   a.logits = c->logits; a.R = B; a.V = c->V; a.k = c->k;
   a.topk = c->st.s1_topk; a.status = c->st.status;
-  timed(c, K_ROWSTATS, 0, 0, [&] { launch_row_stats(a, c->stream); });
+  timed(c, K_ROWSTATS, 0, 0, [&] {
+      a.stamp = c->cur_stamp;
+      launch_row_stats(a, c->stream);
+    });
   timed(c, K_STEPLOGIC, 0, 0, [&] {
     launch_select_s1(c->st, c->tgt.kv, c->dft.kv, c->ss_a, c->ss_hw, c->tcfg.d_model, c->R_pad,
                      c->tcfg.norm_eps, c->stream);
@@ -882,39 +927,102 @@ int32_t cdsl_select(cdsl_ctx* c, int32_t* d_beam, int32_t* d_state, int32_t* d_e
   return CDSL_OK;
 }
 
+}  // extern "C"
+
+namespace {
+
+// Capture one whole step (lookahead, verify, select) into an executable graph.
+int capture_step(cdsl_ctx* c, cudaGraphExec_t* out, long long* nodes_out) {
+  cudaGraph_t g = nullptr;
+  if (cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+    return fail(c, CDSL_ECUDA, "cudaStreamBeginCapture failed");
+  do_lookahead(c);
+  do_verify(c);
+  do_select(c);
+  cudaError_t ce = cudaStreamEndCapture(c->stream, &g);
+  if (ce != cudaSuccess) return fail(c, CDSL_ECUDA, std::string("capture: ") + cudaGetErrorString(ce));
+  size_t nodes = 0;
+  cudaGraphGetNodes(g, nullptr, &nodes);
+  if (nodes_out) *nodes_out = (long long)nodes;
+  ce = cudaGraphInstantiate(out, g, 0);
+  cudaGraphDestroy(g);
+  if (ce != cudaSuccess) {
+    *out = nullptr;
+    return fail(c, CDSL_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
+  }
+  return CDSL_OK;
+}
+
+// Fold the stamped step's launch records into the per-launch totals. Launches are taken in
+// stream order; each is charged from its first block's entry, or from the latest exit of the
+// launches before it when it started earlier (programmatic dependent launch overlaps a
+// kernel's prologue with its predecessor's tail), to its last block's exit. The charged
+// intervals are disjoint, so their sum never exceeds the step's span. Launches without a
+// record (the small step kernels) are charged nothing.
+int fold_stamps(cdsl_ctx* c) {
+  const size_t L = std::min(c->st_recs.size(), (size_t)kStampStride);
+  std::vector<unsigned long long> h((size_t)3 * kStampStride);
+  for (int w = 0; w < 3; ++w)
+    if (cudaMemcpy(h.data() + (size_t)w * kStampStride, c->stamps + (size_t)w * kStampStride,
+                   L * sizeof(unsigned long long), cudaMemcpyDeviceToHost) != cudaSuccess)
+      return cuda_check(c, "cdsl_step (stamps)");
+  c->st_ms.resize(c->st_recs.size(), 0.0);
+  c->st_kbytes.resize(c->st_recs.size(), 0.0);
+  unsigned long long prev_end = 0, first = ~0ull, last = 0;
+  for (size_t i = 0; i < L; ++i) {
+    const unsigned long long t0 = h[i], t1 = h[kStampStride + i];
+    if (t0 == ~0ull || t1 == 0 || t1 < t0) continue;   // no record written
+    first = std::min(first, t0);
+    last = std::max(last, t1);
+    const unsigned long long from = std::max(t0, prev_end);
+    if (t1 > from) c->st_ms[i] += (double)(t1 - from) * 1e-6;
+    prev_end = std::max(prev_end, t1);
+    c->st_kbytes[i] += (double)h[2 * (size_t)kStampStride + i];
+  }
+  if (last > first) c->st_span_ms += (double)(last - first) * 1e-6;
+  c->st_steps += 1;
+  return CDSL_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
 int32_t cdsl_step(cdsl_ctx* c, int32_t* d_beam, int32_t* d_state, int32_t* d_emitted,
                   int32_t* d_n_emitted, float* d_reward) {
   if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
   if (c->phase != PH_READY) return fail(c, CDSL_ESTATE, "cdsl_step needs a prefilled context");
   cudaGetLastError();
-  if (c->stream == nullptr || c->profiling) {  // legacy stream / timing: launch directly
+  bool stamped = false;
+  if (c->stream == nullptr || c->profiling) {  // legacy stream / event timing: launch directly
     do_lookahead(c);
     do_verify(c);
     do_select(c);
+  } else if (c->prof_mode == 2) {             // in-graph timing: the stamped graph
+    if (!c->graph_st) {
+      c->stamping = true;
+      c->st_recs.clear();
+      const int e = capture_step(c, &c->graph_st, nullptr);
+      c->stamping = false;
+      if (e) return e;
+    }
+    const size_t n = sizeof(unsigned long long) * kStampStride;
+    cudaMemsetAsync(c->stamps, 0xff, n, c->stream);
+    cudaMemsetAsync(c->stamps + kStampStride, 0, 2 * n, c->stream);
+    cudaGraphLaunch(c->graph_st, c->stream);
+    stamped = true;
   } else {
     if (!c->graph) {
-      cudaGraph_t g = nullptr;
-      if (cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
-        return fail(c, CDSL_ECUDA, "cudaStreamBeginCapture failed");
-      do_lookahead(c);
-      do_verify(c);
-      do_select(c);
-      cudaError_t ce = cudaStreamEndCapture(c->stream, &g);
-      if (ce != cudaSuccess) return fail(c, CDSL_ECUDA, std::string("capture: ") + cudaGetErrorString(ce));
-      size_t nodes = 0;
-      cudaGraphGetNodes(g, nullptr, &nodes);
-      c->graph_nodes = (long long)nodes;
-      ce = cudaGraphInstantiate(&c->graph, g, 0);
-      cudaGraphDestroy(g);
-      if (ce != cudaSuccess) {
-        c->graph = nullptr;
-        return fail(c, CDSL_ECUDA, std::string("graph instantiate: ") + cudaGetErrorString(ce));
-      }
+      const int e = capture_step(c, &c->graph, &c->graph_nodes);
+      if (e) return e;
     }
     cudaGraphLaunch(c->graph, c->stream);
   }
   copy_select_outputs(c, d_beam, d_state, d_emitted, d_n_emitted, d_reward);
-  return cuda_check(c, "cdsl_step");
+  int e = cuda_check(c, "cdsl_step");
+  if (e || !stamped) return e;
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return cuda_check(c, "cdsl_step");
+  return fold_stamps(c);
 }
 
 int32_t cdsl_get_tokens(cdsl_ctx* c, int32_t* d_tokens, int32_t* d_lengths) {
@@ -940,9 +1048,15 @@ int32_t cdsl_get_counters(cdsl_ctx* c, int64_t* h_counters) {
 
 int32_t cdsl_profile(cdsl_ctx* c, int32_t enable) {
   if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
-  c->profiling = enable != 0;
+  if (enable < 0 || enable > 2) return fail(c, CDSL_EINVAL, "cdsl_profile: mode must be 0, 1 or 2");
+  c->prof_mode = enable;
+  c->profiling = enable == 1;
   c->ev_used = 0;
   c->prof.clear();
+  std::fill(c->st_ms.begin(), c->st_ms.end(), 0.0);
+  std::fill(c->st_kbytes.begin(), c->st_kbytes.end(), 0.0);
+  c->st_steps = 0;
+  c->st_span_ms = 0;
   return CDSL_OK;
 }
 
@@ -951,11 +1065,26 @@ int32_t cdsl_get_profile(cdsl_ctx* c, int32_t impl, double* h_out) {
   cudaError_t e = cudaStreamSynchronize(c->stream);
   if (e != cudaSuccess) return fail(c, CDSL_ECUDA, std::string("cdsl_get_profile: ") + cudaGetErrorString(e));
   double n = 0, ms = 0, by = 0, fl = 0;
-  for (const auto& r : c->prof) {
-    if (r.impl != impl) continue;
-    float t = 0;
-    cudaEventElapsedTime(&t, c->ev_pool[r.ev], c->ev_pool[r.ev + 1]);
-    n += 1; ms += t; by += r.bytes; fl += r.flops;
+  if (c->prof_mode == 2) {
+    const double steps = c->st_steps;
+    if (impl == K_CLASSES) {   // the stamped steps themselves
+      n = steps;
+      ms = c->st_span_ms;
+    }
+    for (size_t i = 0; i < c->st_recs.size() && i < c->st_ms.size(); ++i) {
+      const auto& r = c->st_recs[i];
+      if (r.impl != impl) continue;
+      n += steps; ms += c->st_ms[i];
+      by += r.bytes > 0 ? r.bytes * steps : c->st_kbytes[i];
+      fl += r.flops * steps;
+    }
+  } else {
+    for (const auto& r : c->prof) {
+      if (r.impl != impl) continue;
+      float t = 0;
+      cudaEventElapsedTime(&t, c->ev_pool[r.ev], c->ev_pool[r.ev + 1]);
+      n += 1; ms += t; by += r.bytes; fl += r.flops;
+    }
   }
   h_out[0] = n; h_out[1] = ms; h_out[2] = by; h_out[3] = fl;
   return cuda_check(c, "cdsl_get_profile");
@@ -967,6 +1096,19 @@ int32_t cdsl_get_profile_launches(cdsl_ctx* c, double* h_out, int32_t h_capacity
   if (e != cudaSuccess)
     return -fail(c, CDSL_ECUDA, std::string("cdsl_get_profile_launches: ") + cudaGetErrorString(e));
   int32_t n = 0;
+  if (c->prof_mode == 2) {   // per launch of the stamped step, averaged over the steps
+    const double steps = std::max(1, c->st_steps);
+    for (size_t i = 0; i < c->st_recs.size() && i < c->st_ms.size(); ++i) {
+      if (n >= h_capacity) break;
+      const auto& r = c->st_recs[i];
+      h_out[4 * n] = r.impl;
+      h_out[4 * n + 1] = c->st_ms[i] / steps;
+      h_out[4 * n + 2] = r.bytes > 0 ? r.bytes : c->st_kbytes[i] / steps;
+      h_out[4 * n + 3] = r.flops;
+      ++n;
+    }
+    return n;
+  }
   for (const auto& r : c->prof) {
     if (n >= h_capacity) break;
     float t = 0;
@@ -1004,6 +1146,7 @@ const char* cdsl_last_error(const cdsl_ctx* c) {
 void cdsl_destroy(cdsl_ctx* c) {
   if (!c) return;
   if (c->graph) cudaGraphExecDestroy(c->graph);
+  if (c->graph_st) cudaGraphExecDestroy(c->graph_st);
   for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
   delete c;
 }

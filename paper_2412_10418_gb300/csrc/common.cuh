@@ -102,6 +102,32 @@ template <> __device__ __forceinline__ float load_act<__nv_bfloat16>(const __nv_
   return __bfloat162float(buf[i]) + __bfloat162float(buf[plane + i]);
 }
 
+// Device wall clock in nanoseconds (%globaltimer).
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// In-graph launch timing (cdsl_profile mode 2). A launch's record is three 64-bit words
+// kStampStride apart: [0] the first block's entry, [1] the last block's exit (globaltimer ns,
+// reset to ~0 and 0 before each step), [2] bytes the kernel counted itself (attention), or 0.
+// Thread 0 of every block stamps its entry when constructed and its exit when destroyed.
+constexpr int kStampStride = 16384;   // launches per stamped step, at most
+struct LaunchStamp {
+  unsigned long long* p;
+  __device__ __forceinline__ explicit LaunchStamp(unsigned long long* rec)
+      : p(threadIdx.x == 0 && threadIdx.y == 0 ? rec : nullptr) {
+    if (p) atomicMin(p, (unsigned long long)globaltimer_ns());
+  }
+  __device__ __forceinline__ ~LaunchStamp() {
+    if (p) atomicMax(p + kStampStride, (unsigned long long)globaltimer_ns());
+  }
+  __device__ __forceinline__ void add_bytes(unsigned long long b) const {
+    if (p) atomicAdd(p + 2 * kStampStride, b);
+  }
+};
+
 // Device status word: first error wins, later ones are dropped.
 __device__ __forceinline__ void set_status(int32_t* status, int32_t code) {
   if (status) atomicCAS(status, 0, code);

@@ -59,6 +59,7 @@ struct GemmArgs {
   float* out_ss;           // [ld_out / 32][ld_ss]
   const float* head_w;     // reward head vector [ld_out] (last target layer only), or nullptr
   float* out_hw;           // [ld_out / 32][ld_ss] partial sums of head_w . g . h
+  unsigned long long* stamp;  // in-graph launch timing record (LaunchStamp), or nullptr
 };
 
 // Row scale rsqrt(mean(h^2) + eps) from the 32-feature partial sums of row r. The partials

@@ -14,6 +14,7 @@ constexpr int TV = 128, TR = 32, TK = 32;
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_gemm_simt(GemmArgs a) {
+  const LaunchStamp stamp(a.stamp);
   pdl_wait();
   pdl_launch_dependents();
   __shared__ float Ws[TK][TV + 1];

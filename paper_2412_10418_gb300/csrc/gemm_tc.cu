@@ -83,6 +83,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     k_gemm_tc(const __grid_constant__ TcMaps maps, const __grid_constant__ GemmArgs a, TcPlan p,
               float* part, int* tile_cnt) {
   extern __shared__ uint8_t smem_raw[];
+  const LaunchStamp stamp(a.stamp);
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
   __shared__ __align__(8) uint64_t accf_bar[2];

@@ -1,5 +1,7 @@
-// gemv_stream.cu -- weight-streaming GEMM for few activation rows (the draft decode calls:
-// B*k beam rows, plus one pending row per prompt in the first call).
+// gemv_stream.cu -- CUDA-core weight-streaming GEMM for few activation rows (R <= 8): the
+// projections of bf16 models whose K the tensor-core kernel does not take (K % 64 != 0), and
+// cdsl_gemv_noalloc. Every bf16 projection with K % 64 == 0 -- all of the synthetic workloads'
+// -- runs on the tensor-core kernel (gemm_tc.cu) instead, which streams weights faster here.
 //
 // With R <= 8 rows a projection moves ~R*2 flops per weight byte: the kernel is bound by HBM
 // bandwidth on the weights. Each block owns a tile of 128 virtual output rows and one K slice
@@ -72,6 +74,7 @@ __device__ __forceinline__ void transpose_reduce(float (&v)[NV]) {
 template <int RM>
 __global__ void __launch_bounds__(THREADS) k_gemv(GemmArgs a, int k_split, int n_splits,
                                                  float* part, int* tile_cnt) {
+  const LaunchStamp stamp(a.stamp);
   pdl_wait();
   pdl_launch_dependents();
   extern __shared__ float4 smem4[];

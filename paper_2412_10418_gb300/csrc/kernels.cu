@@ -112,6 +112,7 @@ constexpr int RS_THREADS = 512;
 constexpr int RS_MAXV = 16;   // float4 per thread: V <= 16 * 4 * 512 = 32768
 
 __global__ void __launch_bounds__(RS_THREADS) k_row_stats(RowStatsArgs a) {
+  const LaunchStamp stamp(a.stamp);
   pdl_wait();
   pdl_launch_dependents();
   __shared__ unsigned long long redk[kMaxWarps];

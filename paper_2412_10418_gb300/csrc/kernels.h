@@ -72,6 +72,7 @@ struct AttnArgs {
   int32_t n_chunks, n_tchunks, qb_count, qblock;
   const int32_t* zmap;
   int32_t* status;
+  unsigned long long* stamp;   // in-graph launch timing record (LaunchStamp), or nullptr
 };
 int attn_chunk();
 int attn_max_chunks();
@@ -98,6 +99,7 @@ struct RowStatsArgs {
   int32_t* status;
   // verify: reward head sigmoid(w . RMSNorm(h)) from the last layer's partial sums
   const float* ss; const float* hw; int32_t norm_D, ld_ss; float norm_eps; float* head_out;
+  unsigned long long* stamp;   // in-graph launch timing record (LaunchStamp), or nullptr
 };
 void launch_row_stats(const RowStatsArgs& a, cudaStream_t s);
 
