@@ -49,6 +49,10 @@ def parse():
     ap.add_argument("--verify-sweep", action="store_true",
                     help="time one cdsl_verify + cdsl_select per (k, d, prefix) point of the "
                          "7B-shape verify sweep instead of the step benchmark")
+    ap.add_argument("--sweep-k", default="2,4,8,16", help="verify sweep: beam counts k")
+    ap.add_argument("--sweep-d", default="2,4,6,8,10", help="verify sweep: lookahead lengths d")
+    ap.add_argument("--sweep-prefix", default="512,1024,2048,4096",
+                    help="verify sweep: prefix lengths")
     ap.add_argument("--oracle-layers", type=int, default=2,
                     help="target layers the oracle sample runs (scaled to the full depth)")
     ap.add_argument("--draft-equals-target", action="store_true",
@@ -716,10 +720,11 @@ def verify_sweep(args):
         eng.close()
         return sorted(ts)[len(ts) // 2]
 
-    for prefix in (512, 1024, 2048, 4096):
+    ints = lambda txt: [int(x) for x in txt.split(",") if x]
+    for prefix in ints(args.sweep_prefix):
         t_dec = time_point(1, 1, prefix)
-        for k in (2, 4, 8, 16):
-            for d in (2, 4, 6, 8, 10):
+        for k in ints(args.sweep_k):
+            for d in ints(args.sweep_d):
                 us = time_point(k, d, prefix)
                 rows = k * (d + 1)
                 flops = 2.0 * wl0.target.n_params() * rows

@@ -230,6 +230,17 @@ CDSL_API int32_t cdsl_get_profile_launches(cdsl_ctx* ctx, double* h_out, int32_t
  * d_need = 1). Any pointer may be NULL. CDSL_EINVAL with a smaller budget. */
 CDSL_API int32_t cdsl_get_step1(cdsl_ctx* ctx, int32_t* d_need, int32_t* d_tokens, float* d_reward);
 
+/* Limit of the tensor-core kernels' bounded waits on another agent's progress (a pipeline
+ * stage, an accumulator, an MMA result), in nanoseconds of device wall time; 2 s after
+ * cdsl_init. A wait that runs out latches CDSL_ETIMEOUT in the device status word; the block
+ * then skips the rest of its work, waits (with a fixed 2 s limit) for its own copies and
+ * MMAs in flight, meets its cluster barriers and exits, so the launch ends and the CUDA
+ * context stays usable. The context's results are undefined after CDSL_ETIMEOUT: destroy it
+ * (a new context on the same device works). A short limit exercises that failure path
+ * without a fault (0: every wait not already satisfied gives up). Synchronizes the stream;
+ * the next cdsl_step captures its graph again. */
+CDSL_API int32_t cdsl_set_wait_limit(cdsl_ctx* ctx, uint64_t ns);
+
 /* Synchronize the stream and return the device status word (a cdsl_status; CDSL_OK when no
  * device-side error was latched) in *h_device_status. Clears nothing. */
 CDSL_API int32_t cdsl_get_status(cdsl_ctx* ctx, int32_t* h_device_status);

@@ -70,6 +70,7 @@ EXPORTS = {
     "cdsl_get_profile": (_I, [_P, _I, ctypes.POINTER(ctypes.c_double)]),
     "cdsl_get_profile_launches": (_I, [_P, ctypes.POINTER(ctypes.c_double), _I]),
     "cdsl_gemv_noalloc": (_I, [_P, _I, _I, _P, _I, _P, _P]),
+    "cdsl_set_wait_limit": (_I, [_P, ctypes.c_uint64]),
     "cdsl_last_error": (ctypes.c_char_p, [_P]),
     "cdsl_destroy": (None, [_P]),
 }
@@ -185,6 +186,11 @@ def cdsl_get_counters(ctx) -> List[int]:
 
 def cdsl_get_step1(ctx, need=None, tokens=None, reward=None):
     _check(lib().cdsl_get_step1(ctx, _ptr(need), _ptr(tokens), _ptr(reward)), ctx)
+
+
+def cdsl_set_wait_limit(ctx, ns: int):
+    """Limit (nanoseconds) of the tensor-core kernels' bounded waits; see include/cdsl.h."""
+    _check(lib().cdsl_set_wait_limit(ctx, int(ns)), ctx)
 
 
 def cdsl_get_status(ctx) -> int:

@@ -85,6 +85,7 @@ struct cdsl_ctx {
   int phase = PH_NEW;
   cudaGraphExec_t graph = nullptr;
   long long graph_nodes = 0;
+  uint64_t wait_ns = 2000000000ull;   // limit of the tensor-core kernels' pipeline waits
   // kernel timing (cdsl_profile): mode 1 events around direct launches, mode 2 in-graph stamps
   struct ProfRec { int impl; double bytes, flops; size_t ev; };
   int prof_mode = 0;
@@ -447,6 +448,7 @@ GemmArgs gemm_base(const cdsl_ctx* c, const ModelW& m, int mode, int K, const vo
   a.n_heads = m.cfg.n_heads;
   a.kv = m.kv;
   a.status = c->st.status;
+  a.wait_ns = c->wait_ns;
   return a;
 }
 
@@ -460,6 +462,10 @@ const CUtensorMap& tensor_map(cdsl_ctx* c, const void* base, int inner, int oute
   if (e && !c->map_error) c->map_error = e;
   return c->maps.emplace(key, m).first->second;
 }
+
+// Query vectors per prompt and KV head from which a dense pass of a bf16 model runs on the
+// tensor-core attention (attention_tc.cu) rather than the CUDA-core one (attention.cu).
+constexpr int kAttnTcMinVectors = 128;
 
 // One forward pass of a model over R rows described by `rows`; for lm_rows > 0 the final
 // norm + LM head run over rows gather[i] (or the first lm_rows rows) into logits.
@@ -488,8 +494,17 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
   at.n_chunks = ap.n_chunks ? ap.n_chunks : c->attn_chunks;
   at.n_tchunks = ap.n_tchunks;
   at.status = c->st.status;
+  at.wait_ns = c->wait_ns;
   int n_z;
-  if (ap.zmap) {
+  // dense passes of bf16 models with many query vectors per KV head on the tensor-core
+  // attention (kAttnTcMinVectors)
+  const bool attn_tc = c->dtype == CDSL_DTYPE_BF16 && !ap.zmap &&
+                       ap.rows_per_prompt * (H / KVH) >= kAttnTcMinVectors;
+  if (attn_tc) {
+    at.qblock = attn_tc_qblock(ap.rows_per_prompt, at.G);
+    at.qb_count = (ap.rows_per_prompt * at.G + at.qblock - 1) / at.qblock;
+    n_z = c->B * at.qb_count;
+  } else if (ap.zmap) {
     n_z = (int)ap.zmap->size() / 2;
     at.zmap = c->attn_zmap;
     at.qblock = attn_qblock();
@@ -528,7 +543,8 @@ void forward(cdsl_ctx* c, ModelW& m, const RowDesc* rows, int R, int lm_rows,
     at.layer = l;
     timed(c, K_ATTN, 0, 0, [&] {
       at.stamp = c->cur_stamp;
-      launch_attn(c->dtype, at, n_z, s);
+      if (attn_tc) launch_attn_tc(at, n_z, s);
+      else launch_attn(c->dtype, at, n_z, s);
       at.stamp = nullptr;
     });
     GemmArgs o = gemm_base(c, m, EPI_RESID, H * hd, c->Xa, H * hd, R);
@@ -763,6 +779,10 @@ int32_t cdsl_init(const cdsl_model_cfg* target, const void* const* h_target_weig
   if (configure_attention()) {
     delete c;
     return fail(nullptr, CDSL_ECUDA, "cannot configure the attention kernel (shared memory)");
+  }
+  if (c->dtype == CDSL_DTYPE_BF16 && configure_attention_tc()) {
+    delete c;
+    return fail(nullptr, CDSL_ECUDA, "cannot configure the tensor-core attention (shared memory)");
   }
   if (c->dtype == CDSL_DTYPE_BF16 && configure_gemm_tc()) {
     delete c;
@@ -1117,6 +1137,17 @@ int32_t cdsl_get_profile_launches(cdsl_ctx* c, double* h_out, int32_t h_capacity
     ++n;
   }
   return n;
+}
+
+int32_t cdsl_set_wait_limit(cdsl_ctx* c, uint64_t ns) {
+  if (!c) return fail(nullptr, CDSL_EINVAL, "ctx is NULL");
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return cuda_check(c, "cdsl_set_wait_limit");
+  c->wait_ns = ns;
+  // the step graphs hold the old limit in their kernel arguments: capture them again
+  if (c->graph) cudaGraphExecDestroy(c->graph);
+  if (c->graph_st) cudaGraphExecDestroy(c->graph_st);
+  c->graph = c->graph_st = nullptr;
+  return CDSL_OK;
 }
 
 int32_t cdsl_get_step1(cdsl_ctx* c, int32_t* d_need, int32_t* d_tokens, float* d_reward) {

@@ -22,6 +22,7 @@
 
 #include <cooperative_groups.h>
 
+#include "attn_layout.cuh"
 #include "kernels.h"
 
 namespace cdsl {
@@ -29,12 +30,11 @@ namespace {
 
 namespace cg = cooperative_groups;
 
-constexpr int ACH = 64;              // key slots per chunk
+using attn::ACH;
+using attn::MAXP;
+using attn::MAXCB;
 constexpr int AQB = 40;              // query vectors per cluster (at most)
-constexpr int MAXP = 128;            // chunks (prefix + tail) of a pass
 constexpr int ACL = 16;              // blocks per cluster (at most)
-constexpr int MAXCB = MAXP / 8;      // chunks per block (at most; clusters have >= 8 blocks
-                                     // whenever a pass has more than 8 chunks)
 constexpr int ATHREADS = 256;
 constexpr int AWARPS = ATHREADS / 32;
 
@@ -50,23 +50,17 @@ struct AttnSmem {
 
 template <typename T, int HD, int QPW>
 __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
-  using L = AttnSmem<HD>;
+  const LaunchStamp stamp(a.stamp);
+  using SL = AttnSmem<HD>;
   constexpr int QB = AWARPS * QPW;              // query vectors of the cluster
   extern __shared__ float4 sm4[];
   float* qS = reinterpret_cast<float*>(sm4);   // [QB][QP]  pre-scaled queries
-  float* kS = qS + AQB * L::QP;                 // [ACH][QP]; after the chunks: partial o [QB][HD]
-  float* vS = kS + ACH * L::QP;                 // [ACH][HD]
+  float* kS = qS + AQB * SL::QP;                 // [ACH][QP]; after the chunks: partial o [QB][HD]
+  float* vS = kS + ACH * SL::QP;                 // [ACH][HD]
   float* pS = vS + ACH * HD;                    // [ACH][PP] probabilities
-  __shared__ int s_row[QB], s_gg[QB], s_np[QB], s_tb[QB], s_nt[QB];
-  __shared__ int s_toff[32], s_tlen[32], s_ttb[32];   // per row of the block: its tail's
-                                                      // slot range (first row of a tail only)
-  __shared__ int s_wcnt[AWARPS];
-  __shared__ int s_nrows, s_maxnp;
+  __shared__ attn::Layout<QB> L;
+  __shared__ int s_nkeys;
   __shared__ float s_pm[QB], s_pl[QB];          // the block's partial (m, l) per query vector
-  __shared__ int s_kslot[MAXCB * ACH];          // every key slot of the block's chunks: the page
-                                                // (prefix chunk) or tail row (tail chunk), -1 empty
-  __shared__ int s_ktb[MAXCB * ACH];            // tail slots: tail base of the beam,
-  __shared__ uint8_t s_kj[MAXCB * ACH];         //   index in it
 
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)gridDim.x;                 // = cluster size
@@ -85,102 +79,12 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   const int G = a.G, H = a.n_heads;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  // ---- this cluster's query vectors: rows of prompt b in order, G heads each. The rows (plan
-  //      kernel), the committed page table and the tail layout come from kernels the launch
-  //      chain has already completed, so everything up to the key slots precedes the wait.
-  if (threadIdx.x < QB) s_row[threadIdx.x] = -1;
-  for (int i = threadIdx.x; i < MAXCB * ACH; i += ATHREADS) s_kslot[i] = -1;
-  if (threadIdx.x == 0) s_nrows = 0;
-  __syncthreads();
-  for (int base = 0; base < a.R; base += ATHREADS) {
-    const int r = base + threadIdx.x;
-    RowDesc rd;
-    const bool mine = r < a.R && (rd = a.rows[r]).b == b;
-    const unsigned bal = __ballot_sync(0xffffffffu, mine);
-    if (lane == 0) s_wcnt[warp] = __popc(bal);
-    __syncthreads();
-    int off = s_nrows;
-    for (int w = 0; w < warp; ++w) off += s_wcnt[w];
-    const int local = off + __popc(bal & ((1u << lane) - 1));
-    if (mine) {
-      for (int gg = 0; gg < G; ++gg) {
-        const int qi = local * G + gg - qb * QB;
-        if (qi >= 0 && qi < QB) {
-          s_row[qi] = r;
-          s_gg[qi] = gg;
-          s_np[qi] = rd.n_prefix;
-          s_tb[qi] = rd.tail_base;
-          s_nt[qi] = rd.n_tail;
-        }
-      }
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      int tot = 0;
-      for (int w = 0; w < AWARPS; ++w) tot += s_wcnt[w];
-      s_nrows += tot;
-    }
-    __syncthreads();
-  }
-  const int nq = max(0, min(QB, s_nrows * G - qb * QB));
-  if (warp == 0) {
-    // longest prefix, and the distinct tails (lane = row of the block: at most 32, see
-    // attn_qblock_for) in order of first appearance, each as long as its longest row: slot
-    // offsets in their concatenation
-    const int first_local = (qb * QB) / G;
-    const int qi_l = max(0, (first_local + lane) * G - qb * QB);   // the row's first vector
-    const bool row_ok = nq > 0 && qi_l < nq && lane <= (qb * QB + nq - 1) / G - first_local;
-    int np = row_ok ? s_np[qi_l] : 0;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) np = max(np, __shfl_xor_sync(0xffffffffu, np, o));
-    const int tb = row_ok ? s_tb[qi_l] : -1;
-    const int nt = row_ok ? s_nt[qi_l] : 0;
-    int len = 0;
-    bool first = nt > 0;
-    for (int j = 0; j < 32; ++j) {
-      const int tbj = __shfl_sync(0xffffffffu, tb, j), ntj = __shfl_sync(0xffffffffu, nt, j);
-      if (tbj == tb && ntj > 0) {
-        len = max(len, ntj);
-        if (j < lane) first = false;
-      }
-    }
-    if (!first) len = 0;
-    int off = len;   // inclusive scan of the lengths over the lanes
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, off, o);
-      if (lane >= o) off += v;
-    }
-    const int total = __shfl_sync(0xffffffffu, off, 31);
-    s_toff[lane] = off - len;
-    s_tlen[lane] = len;
-    s_ttb[lane] = tb;
-    if (lane == 0) {
-      s_maxnp = np;
-      if (cx == 0 && total > a.n_tchunks * ACH) set_status(a.status, CDSL_ERANGE);
-    }
-  }
-  __syncthreads();
-  const int maxnp = s_maxnp;
-  // key slots of this block's chunks
-  for (int i = 0; i < nb_chunks; ++i) {
-    const int c = cx + i * C;
-    if (c < n_p) {   // prefix positions c*64 .. c*64 + 63 below the longest prefix
-      const int t = c * ACH + (threadIdx.x & (ACH - 1));
-      if (threadIdx.x < ACH && t < maxnp) {
-        s_kslot[i * ACH + threadIdx.x] = a.kv.page_table[b * a.kv.max_pages + (t >> a.kv.page_shift)];
-      }
-    } else if (warp == 0) {   // tail slots [lo, lo + 64) of the concatenation
-      const int lo = (c - n_p) * ACH, off = s_toff[lane], len = s_tlen[lane], tb = s_ttb[lane];
-      for (int e = max(0, lo - off); e < len && off + e < lo + ACH; ++e) {
-        const int sl = i * ACH + off + e - lo;
-        s_kslot[sl] = tb + e;
-        s_ktb[sl] = tb;
-        s_kj[sl] = (uint8_t)e;
-      }
-    }
-  }
-  __syncthreads();
+  // ---- this cluster's query vectors and this block's key slots. The rows (plan kernel), the
+  //      committed page table and the tail layout come from kernels the launch chain has
+  //      already completed, so all of it precedes the wait.
+  const int nq = attn::build_layout<QB, ATHREADS>(L, a, b, qb, cx, C, nb_chunks);
+  const int maxnp = L.maxnp;
+  if (a.stamp) attn::count_bytes<QB, ATHREADS, HD>(L, stamp, qb, cx, nb_chunks, nq, &s_nkeys);
   pdl_wait();                 // q and K/V of the previous kernels are ready
   pdl_launch_dependents();
 
@@ -215,15 +119,15 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
         qr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
         if (qi < nq && qi < QB)
-          qr[u] = *reinterpret_cast<const float4*>(a.q + (size_t)s_row[qi] * H * HD +
-                                                   (size_t)(g * G + s_gg[qi]) * HD + 4 * e4);
+          qr[u] = *reinterpret_cast<const float4*>(a.q + (size_t)L.row[qi] * H * HD +
+                                                   (size_t)(g * G + L.gg[qi]) * HD + 4 * e4);
       }
     }
 #pragma unroll
     for (int u = 0; u < PER; ++u) {
       const int idx = threadIdx.x + u * ATHREADS;
       const int j = idx / (HD / 4), e4 = idx % (HD / 4);
-      const int ks = s_kslot[i * ACH + j];
+      const int ks = L.kslot[i * ACH + j];
       kr[u] = vr[u] = make_float4(0.f, 0.f, 0.f, 0.f);
       if (ks >= 0) {
         const float* kp = tail ? a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, ks, g)
@@ -241,7 +145,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
         const int qi = idx / (HD / 4), e4 = idx % (HD / 4);
         float4 v = qr[u];
         v.x *= a.scale; v.y *= a.scale; v.z *= a.scale; v.w *= a.scale;
-        if (qi < QB) *reinterpret_cast<float4*>(qS + qi * L::QP + 4 * e4) = v;
+        if (qi < QB) *reinterpret_cast<float4*>(qS + qi * SL::QP + 4 * e4) = v;
       }
       q_staged = true;
     }
@@ -249,7 +153,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     for (int u = 0; u < PER; ++u) {
       const int idx = threadIdx.x + u * ATHREADS;
       const int j = idx / (HD / 4), e4 = idx % (HD / 4);
-      *reinterpret_cast<float4*>(kS + j * L::QP + 4 * e4) = kr[u];
+      *reinterpret_cast<float4*>(kS + j * SL::QP + 4 * e4) = kr[u];
       *reinterpret_cast<float4*>(vS + j * HD + 4 * e4) = vr[u];
     }
     __syncthreads();
@@ -261,11 +165,11 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     for (int q = 0; q < QPW; ++q) s[q][0] = s[q][1] = 0.f;
 #pragma unroll 4
     for (int e = 0; e < HD; e += 4) {
-      const float4 k0 = *reinterpret_cast<const float4*>(kS + lane * L::QP + e);
-      const float4 k1 = *reinterpret_cast<const float4*>(kS + (lane + 32) * L::QP + e);
+      const float4 k0 = *reinterpret_cast<const float4*>(kS + lane * SL::QP + e);
+      const float4 k1 = *reinterpret_cast<const float4*>(kS + (lane + 32) * SL::QP + e);
 #pragma unroll
       for (int q = 0; q < QPW; ++q) {
-        const float4 qv = *reinterpret_cast<const float4*>(qS + (q0 + q) * L::QP + e);
+        const float4 qv = *reinterpret_cast<const float4*>(qS + (q0 + q) * SL::QP + e);
         s[q][0] += qv.x * k0.x + qv.y * k0.y + qv.z * k0.z + qv.w * k0.w;
         s[q][1] += qv.x * k1.x + qv.y * k1.y + qv.z * k1.z + qv.w * k1.w;
       }
@@ -281,13 +185,13 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
       if (qi >= nq) {
         ok0 = ok1 = false;
       } else if (!tail) {         // prefix: positions before the row's prefix length
-        ok0 = t0 + lane < s_np[qi];
-        ok1 = t0 + lane + 32 < s_np[qi];
+        ok0 = t0 + lane < L.np[qi];
+        ok1 = t0 + lane + 32 < L.np[qi];
       } else {                    // tail: the row's own beam, causal within it
-        const int tb = s_tb[qi], nt = s_nt[qi];
+        const int tb = L.tb[qi], nt = L.nt[qi];
         const int k0 = i * ACH + lane, k1 = k0 + 32;
-        ok0 = s_kslot[k0] >= 0 && s_ktb[k0] == tb && s_kj[k0] < nt;
-        ok1 = s_kslot[k1] >= 0 && s_ktb[k1] == tb && s_kj[k1] < nt;
+        ok0 = L.kslot[k0] >= 0 && L.ktb[k0] == tb && L.kj[k0] < nt;
+        ok1 = L.kslot[k1] >= 0 && L.ktb[k1] == tb && L.kj[k1] < nt;
       }
       s[q][0] = ok0 ? s[q][0] : -INFINITY;   // masked keys: exp(-inf - m) = 0 below
       s[q][1] = ok1 ? s[q][1] : -INFINITY;
@@ -321,17 +225,17 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
       for (int c2 = 0; c2 < DPL; ++c2) o[q][c2] *= alpha[q];
     }
     if constexpr (QPW == 4) {
-      *reinterpret_cast<float4*>(pS + lane * L::PP + q0) = make_float4(p0[0], p0[1], p0[2], p0[3]);
-      *reinterpret_cast<float4*>(pS + (lane + 32) * L::PP + q0) =
+      *reinterpret_cast<float4*>(pS + lane * SL::PP + q0) = make_float4(p0[0], p0[1], p0[2], p0[3]);
+      *reinterpret_cast<float4*>(pS + (lane + 32) * SL::PP + q0) =
           make_float4(p1[0], p1[1], p1[2], p1[3]);
     } else if constexpr (QPW == 2) {
-      *reinterpret_cast<float2*>(pS + lane * L::PP + q0) = make_float2(p0[0], p0[1]);
-      *reinterpret_cast<float2*>(pS + (lane + 32) * L::PP + q0) = make_float2(p1[0], p1[1]);
+      *reinterpret_cast<float2*>(pS + lane * SL::PP + q0) = make_float2(p0[0], p0[1]);
+      *reinterpret_cast<float2*>(pS + (lane + 32) * SL::PP + q0) = make_float2(p1[0], p1[1]);
     } else {
 #pragma unroll
       for (int q = 0; q < QPW; ++q) {
-        pS[lane * L::PP + q0 + q] = p0[q];
-        pS[(lane + 32) * L::PP + q0 + q] = p1[q];
+        pS[lane * SL::PP + q0 + q] = p0[q];
+        pS[(lane + 32) * SL::PP + q0 + q] = p1[q];
       }
     }
     __syncwarp();
@@ -341,14 +245,14 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     for (int t = 0; t < ACH; ++t) {
       float pp[QPW];
       if constexpr (QPW == 4) {
-        const float4 p4 = *reinterpret_cast<const float4*>(pS + t * L::PP + q0);
+        const float4 p4 = *reinterpret_cast<const float4*>(pS + t * SL::PP + q0);
         pp[0] = p4.x; pp[1] = p4.y; pp[2] = p4.z; pp[3] = p4.w;
       } else if constexpr (QPW == 2) {
-        const float2 p2 = *reinterpret_cast<const float2*>(pS + t * L::PP + q0);
+        const float2 p2 = *reinterpret_cast<const float2*>(pS + t * SL::PP + q0);
         pp[0] = p2.x; pp[1] = p2.y;
       } else {
 #pragma unroll
-        for (int q = 0; q < QPW; ++q) pp[q] = pS[t * L::PP + q0 + q];
+        for (int q = 0; q < QPW; ++q) pp[q] = pS[t * SL::PP + q0 + q];
       }
       float v[DPL];
       if constexpr (DPL == 4) {
@@ -429,7 +333,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
     }
     const float inv = Lsum > 0.f ? 1.0f / Lsum : 0.f;
     T* out = reinterpret_cast<T*>(a.out);
-    const size_t dst = (size_t)s_row[qi] * H * HD + (size_t)(g * G + s_gg[qi]) * HD + DPL * lane;
+    const size_t dst = (size_t)L.row[qi] * H * HD + (size_t)(g * G + L.gg[qi]) * HD + DPL * lane;
 #pragma unroll
     for (int c2 = 0; c2 < DPL; ++c2) store_act<T>(out, a.plane, dst + c2, acc[c2] * inv);
   }
@@ -438,7 +342,8 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
 
 template <typename T, int HD, int QPW>
 void launch_t(const AttnArgs& a, int n_z, cudaStream_t s) {
-  const int cl = std::min(g_max_cluster, a.n_chunks + a.n_tchunks);
+  const int cl = attn_cluster_size(g_max_cluster, a.n_chunks + a.n_tchunks, a.kv.kvh * n_z,
+                                   2 * kPlanSMs);
   launch_pdl_cluster(k_attn<T, HD, QPW>, dim3(cl, a.kv.kvh, n_z), dim3(ATHREADS),
                      AttnSmem<HD>::bytes, cl, s, a);
 }
@@ -488,9 +393,10 @@ int attn_qblock_for(int rows_per_prompt, int G) {
 
 int attn_tail_chunks(int rows_per_prompt, int G, int rows_per_tail, int max_tail) {
   if (max_tail <= 0 || rows_per_prompt <= 0) return 0;
-  // rows met by one query block (it may straddle a row at either end), and the distinct
+  // rows met by one query block (at most 32 in either attention kernel), and the distinct
   // tails among them when consecutive runs of rows_per_tail rows share one
-  const int rows = std::min(rows_per_prompt, (AQB + G - 1) / G + 1);
+  (void)G;
+  const int rows = std::min(rows_per_prompt, 32);
   const int tails = std::min(rows, (rows - 1) / std::max(1, rows_per_tail) + 2);
   return (tails * max_tail + ACH - 1) / ACH;
 }

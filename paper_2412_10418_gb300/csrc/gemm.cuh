@@ -48,6 +48,7 @@ struct GemmArgs {
   const RowDesc* rows;     // QKV: per-row position and KV destination
   const float2* rope;      // QKV: [pos][hd/2] (cos, sin)
   int32_t* status;         // device status word (bounded waits report CDSL_ETIMEOUT here)
+  uint64_t wait_ns;        // limit of the tensor-core kernel's pipeline waits (nanoseconds)
   // input normalization: rows are h . g, scale by rsqrt(sum(in_ss[c][r]) / norm_D + eps)
   const float* in_ss;      // [norm_D / 32][ld_ss] partial sums of squares, or nullptr
   int32_t norm_D;

@@ -88,6 +88,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
   __shared__ __align__(8) uint64_t accf_bar[2];
   __shared__ __align__(8) uint64_t acce_bar[2];
+  __shared__ __align__(8) uint64_t drain_bar;   // every MMA this block issued has completed
   __shared__ uint32_t tmem_base;
   __shared__ int s_abort, s_last;
   __shared__ int s_slot_off[kMaxContrib];   // reducer: scratch offset (floats) per contributor
@@ -121,6 +122,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_units = u1 - u0;
   const int pre = min(S, n_units);
   int t_cur = u0 / KBT, kb_cur = u0 % KBT;
+  int n_issued = 0;   // (thread 0) units whose copies were issued
   uint64_t pol = 0;
   auto load_w = [&](int i, int t, int kb) {
     int m0, y0, m1, y1;
@@ -147,6 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc::mbar_init(&accf_bar[i], 1);
       tc::mbar_init(&acce_bar[i], kEpThreads);
     }
+    tc::mbar_init(&drain_bar, 1);
     s_abort = 0;
     tc::fence_mbar_init();
     tc::fence_proxy_async();
@@ -182,7 +185,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       issued = pre;
       for (int i = pre; i < n_units; ++i) {
         const int s = i % S, use = i / S;
-        if (!tc::mbar_wait(&empty_bar[s], (use - 1) & 1, a.status)) {
+        if (!tc::mbar_wait(&empty_bar[s], (use - 1) & 1, a.status, a.wait_ns)) {
           aborted = true;
           break;
         }
@@ -192,11 +195,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (++kb_cur == KBT) { kb_cur = 0; ++t_cur; }
         ++issued;
       }
-      if (aborted) {
-        s_abort = 1;
-        for (int i = max(0, issued - S); i < issued; ++i)
-          tc::mbar_wait(&full_bar[i % S], (i / S) & 1, a.status);
-      }
+      if (aborted) s_abort = 1;
+      n_issued = issued;
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -208,7 +208,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       while (u < u1 && ok) {
         const int seg_end = min(u1, (u / KBT + 1) * KBT);
         const int acc = seg & 1;
-        if (seg >= 2 && !tc::mbar_wait(&acce_bar[acc], ((seg >> 1) - 1) & 1, a.status)) {
+        if (seg >= 2 &&
+            !tc::mbar_wait(&acce_bar[acc], ((seg >> 1) - 1) & 1, a.status, a.wait_ns)) {
           ok = false;
           break;
         }
@@ -217,7 +218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int seg_begin = u;
         for (; u < seg_end; ++u) {
           const int i = (int)(u - u0), s = i % S, use = i / S;
-          if (!tc::mbar_wait(&full_bar[s], use & 1, a.status)) {
+          if (!tc::mbar_wait(&full_bar[s], use & 1, a.status, a.wait_ns)) {
             ok = false;
             break;
           }
@@ -240,10 +241,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc::umma_commit(&empty_bar[s]);
         }
+        if (!ok) break;   // an unfinished accumulator is never handed to the epilogue
         tc::umma_commit(&accf_bar[acc]);
         ++seg;
       }
       if (!ok) s_abort = 1;
+      // every MMA issued here completes before TMEM is released (fixed limit)
+      tc::umma_commit(&drain_bar);
+      tc::mbar_wait(&drain_bar, 0, a.status);
     }
   } else {
     // ---------------- epilogue warps 2..5: TMEM lanes 32*(warp % 4) .. +31
@@ -262,7 +267,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int seg_end = min(u1, (t + 1) * KBT);
       const bool whole = (u % KBT) == 0 && seg_end == (t + 1) * KBT;
       const int acc = seg & 1;
-      if (!tc::mbar_wait(&accf_bar[acc], (seg >> 1) & 1, a.status)) {
+      const bool ready = tc::mbar_wait(&accf_bar[acc], (seg >> 1) & 1, a.status, a.wait_ns);
+      // the epilogue warps give up together or not at all: named barriers and warp-collective
+      // TMEM loads follow
+      if (tc::named_barrier_or(1, kEpThreads, !ready)) {
         s_abort = 1;
         break;
       }
@@ -394,6 +402,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc::tc_fence_before();
   __syncthreads();
+  if (threadIdx.x == 0 && s_abort) {
+    // a block that gave up waits for the copies it issued last to land before it leaves (the
+    // earlier ones were consumed, so they have landed); fixed limit
+    for (int i = max(0, n_issued - S); i < n_issued; ++i)
+      tc::mbar_wait(&full_bar[i % S], (i / S) & 1, a.status);
+  }
   if (warp == 1) tc::tmem_dealloc(tmem, 2 * acc_cols);
 }
 
@@ -465,10 +479,14 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
     p.ctas = p.tiles * S;
     p.ep_rows = p.n_pad;   // the whole partial tile stays in shared memory
     p.stages = fit(budget, p.ep_rows);
-  } else if (cluster < 0 && max_split == 0 && p.tiles <= per_sm * n_sm) {
-    // as many tiles as block slots or fewer, but too many for clusters: one block per whole
-    // tile (no split, no fixup). Measured against stream-K over all 304 slots: 38.4 vs 41.2 us
-    // (7B gate/up), 46.2 vs 55.2 us (7B LM head), 22.8 vs 25.2 us (draft LM head).
+  } else if (cluster < 0 && max_split == 0 && p.tiles <= per_sm * n_sm &&
+             10 * p.tiles >= 9 * n_sm) {
+    // about one tile per SM or more, but too many for clusters: one block per whole tile (no
+    // split, no fixup). Measured against stream-K over all 304 slots: 38.4 vs 41.2 us (7B
+    // gate/up), 46.2 vs 55.2 us (7B LM head), 22.8 vs 25.2 us (draft LM head). With fewer
+    // tiles than that (e.g. the 40-tile projections of the 13B verify pass at 224 rows, whose
+    // partial tiles are too large for clusters) whole tiles would leave most SMs idle:
+    // stream-K over every block slot instead.
     p.ctas = p.tiles;
   }
   p.smem = (size_t)p.stages * stage + (size_t)p.ep_rows * kTileLd * 4 + 1024;

@@ -73,6 +73,7 @@ struct AttnArgs {
   const int32_t* zmap;
   int32_t* status;
   unsigned long long* stamp;   // in-graph launch timing record (LaunchStamp), or nullptr
+  uint64_t wait_ns;            // limit of the tensor-core kernel's MMA waits (nanoseconds)
 };
 int attn_chunk();
 int attn_max_chunks();
@@ -84,6 +85,11 @@ int attn_qblock_for(int rows_per_prompt, int G);
 int attn_tail_chunks(int rows_per_prompt, int G, int rows_per_tail, int max_tail);
 int configure_attention();
 void launch_attn(int dtype, const AttnArgs& a, int n_z, cudaStream_t s);
+// Tensor-core attention (attention_tc.cu) for dense passes of bf16 models (no zmap): query
+// blocks of attn_tc_qblock() vectors (at most 128), head_dim 64 or 128.
+int attn_tc_qblock(int rows_per_prompt, int G);
+int configure_attention_tc();
+void launch_attn_tc(const AttnArgs& a, int n_z, cudaStream_t s);
 // Row statistics of logits rows: argmax (lower id on ties), log-sum-exp, top-k, log p.
 //   draft mode  (dp1 == 0): x[r*out_stride + out_off] = argmax, logq[...] = log q(argmax)
 //   verify mode (dp1 == d+1): amax[r], topk[r, k], logp of the next drafted token

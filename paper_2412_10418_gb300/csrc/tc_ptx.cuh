@@ -11,7 +11,11 @@
 namespace cdsl {
 namespace tc {
 
-// A bounded wait gives up after this many nanoseconds of wall time (device %globaltimer).
+// A bounded wait gives up after a limit of wall time (device %globaltimer). Waits on another
+// agent's progress (a pipeline stage filled or drained, an accumulator finished) take the
+// launch's limit (GemmArgs / AttnArgs wait_ns, 2 s unless cdsl_set_wait_limit changed it);
+// the waits of a block winding down for its own copies and MMAs in flight always take this
+// fixed limit, so that no block leaves while its asynchronous operations still run.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -58,12 +62,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* m, uint32_t parity) {
   return ok != 0;
 }
 // Wait for the phase of parity `parity` to complete; false (and CDSL_ETIMEOUT latched in
-// *status) if it has not after kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait(uint64_t* m, uint32_t parity, int32_t* status) {
+// *status) if it has not after limit_ns.
+__device__ __forceinline__ bool mbar_wait(uint64_t* m, uint32_t parity, int32_t* status,
+                                          uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(m, parity)) return true;
   const uint64_t t0 = globaltimer();
   while (!mbar_try_wait(m, parity)) {
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    if (globaltimer() - t0 > limit_ns) {
       set_status(status, CDSL_ETIMEOUT);
       return false;
     }
@@ -212,9 +217,9 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
                : "memory");
 }
 // Warp-collective load of 16 consecutive fp32 columns of this warp's 32 TMEM lanes
-// (lane i of the warp gets TMEM lane (taddr >> 16) + i).
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
-  uint32_t r[16];
+// (lane i of the warp gets TMEM lane (taddr >> 16) + i), without waiting: the registers are
+// valid after tmem_wait_ld().
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
       "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
@@ -222,9 +227,42 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
+}
+// Wait until every tcgen05.ld this thread issued has completed.
+__device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// Load-and-wait form of tmem_ld16_nowait.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  tmem_ld16_nowait(taddr, r);
+  tmem_wait_ld();
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Warp-collective store of 16 consecutive fp32 columns to this warp's 32 TMEM lanes (lane i
+// of the warp writes TMEM lane (taddr >> 16) + i); waits until the stores have completed.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])),
+      "r"(__float_as_uint(v[3])), "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])),
+      "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])), "r"(__float_as_uint(v[8])),
+      "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+      "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])),
+      "r"(__float_as_uint(v[15]))
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Byte offset of 16-byte chunk `ch` (0..7) of row `r` in a K-major operand tile of 128-byte
+// rows stored with the 128-byte swizzle (the layout TMA's SWIZZLE_128B writes and desc_sw128
+// describes): 8-row atoms of 1024 bytes, chunk index XOR (row mod 8). The tile base must be
+// 1024-byte aligned.
+__device__ __forceinline__ uint32_t sw128_offset(int r, int ch) {
+  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((ch ^ (r & 7)) << 4));
 }
 
 }  // namespace tc
