@@ -571,7 +571,8 @@ def gpu_main(args):
             "achieved": round(a_gbs, 1), "frac": round(a_gbs / hbm, 4),
             "ms_per_step_in_graph": round(att["ms"] / n_prof, 4),
             "bytes": "counted by the kernel: K and V (fp32) of every key once per prompt and "
-                     "KV head, every query vector read and its output written once"}
+                     "KV head, every query vector read and its output written once",
+            "by_shape": by_shape(launches, 3, 1, hbm)[:6]}
     roofline["in_graph_ms_per_step"] = {k: round(v["ms"] / n_prof, 4) for k, v in prof.items()
                                         if v["ms"] > 0}
     # the same launches bracketed by CUDA events outside the graph (no overlap between them)

@@ -101,16 +101,56 @@ __device__ __forceinline__ const T* virtual_row(const GemmArgs& a, int v) {
   return nullptr;
 }
 
+// Items of a tile each epilogue thread works on per pass in the batched epilogues (their loads
+// in flight together).
+constexpr int kEpiBatch = 8;
+
+// What the QKV epilogue needs of one activation row: the RoPE position and where the row's k
+// and v go (element offset of k, head 0 in the prefix pool or the beam tails). A kernel that
+// finishes many tiles over the same rows gathers these once (qkv_rows) instead of every tile
+// reading the row descriptor and the page table again.
+struct QkvRow {
+  int32_t pos;
+  int32_t where;   // 0: not stored, 1: prefix pool, 2: beam tail
+  int64_t base;
+};
+
+// rows[i] for activation rows i < n (by `nthr` threads, tid = 0 .. nthr-1; the caller
+// synchronizes afterwards).
+__device__ __forceinline__ void qkv_rows(const GemmArgs& a, int n, QkvRow* rows, int tid,
+                                         int nthr) {
+  const KvStore& kv = a.kv;
+  for (int r = tid; r < n; r += nthr) {
+    const RowDesc rd = a.rows[r];
+    QkvRow m{rd.pos, 0, 0};
+    if (rd.kv_dst >= 0) {
+      m.where = 2;
+      m.base = (int64_t)kv_tail_offset(kv, a.layer, 0, rd.kv_dst, 0);
+    } else if (rd.kv_dst == KV_PREFIX) {
+      const int page = kv.page_table[rd.b * kv.max_pages + (rd.pos >> kv.page_shift)];
+      if (page >= 0) {
+        m.where = 1;
+        m.base = (int64_t)kv_prefix_offset(kv, a.layer, page, 0, 0,
+                                           rd.pos & ((1 << kv.page_shift) - 1));
+      }
+    }
+    rows[r] = m;
+  }
+}
+
 __device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }
 
 // Apply the epilogue to a finished fp32 tile: tile[r * ldt + v] holds y for activation row
 // r0 + r and virtual row v0 + v (v in [0, 128)), for r in [0, rt). s_rs[r] is the input row
-// scale of row r0 + r when a.in_ss is set (see input_row_scales). Run by `nthr` threads (a
-// multiple of 32; tid = 0 .. nthr-1; all threads of the block by default), which the caller
-// synchronizes before and after.
-template <typename T>
+// scale of row r0 + r when a.in_ss is set (see input_row_scales). kBatch: the residual and
+// QKV epilogues issue kEpiBatch items' loads per thread before their stores (for tiles of many
+// rows); the QKV one then takes the rows' QkvRow from qrows (indexed by row, not r). Run by
+// `nthr` threads (a multiple of 32; tid = 0 .. nthr-1; all threads of the block by default),
+// which the caller synchronizes before and after.
+template <typename T, bool kBatch = false>
 __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const float* tile,
-                              int ldt, const float* s_rs, int tid = -1, int nthr = -1) {
+                              int ldt, const float* s_rs, int tid = -1, int nthr = -1,
+                              const QkvRow* qrows = nullptr) {
   if (tid < 0) {
     tid = threadIdx.x;
     nthr = blockDim.x;
@@ -130,7 +170,7 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
       if (scaled) y *= s_rs[r];
       if (row < R && n < nv) out[(size_t)row * ld + n] = y;
     }
-  } else if (mode == EPI_RESID) {
+  } else if (mode == EPI_RESID && !kBatch) {
     float* __restrict__ const out = a.out_f32;
     const size_t ld = (size_t)a.ld_out, plane = (size_t)a.act_plane, ld_ss = (size_t)a.ld_ss;
     T* const next_x = reinterpret_cast<T*>(a.next_x);
@@ -165,6 +205,54 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
         }
       }
     }
+  } else if (mode == EPI_RESID) {
+    float* __restrict__ const out = a.out_f32;
+    const size_t ld = (size_t)a.ld_out, plane = (size_t)a.act_plane, ld_ss = (size_t)a.ld_ss;
+    T* const next_x = reinterpret_cast<T*>(a.next_x);
+    const T* const next_g = reinterpret_cast<const T*>(a.next_g);
+    float* const out_ss = a.out_ss;
+    const float* const head_w = a.head_w;
+    float* const out_hw = a.out_hw;
+    // kEpiBatch items per thread per pass: every residual load of a pass is issued
+    // before its first store, so a tile of many rows costs rt / kEpiBatch round trips to
+    // memory instead of rt. Every warp sees 32 features of one row (warp_sum below).
+    const int items = rt * 128;
+    for (int base = tid; base < items; base += nthr * kEpiBatch) {
+      float hres[kEpiBatch];
+#pragma unroll
+      for (int u = 0; u < kEpiBatch; ++u) {
+        const int idx = base + u * nthr, r = idx >> 7, v = idx & 127, row = r0 + r, n = v0 + v;
+        hres[u] = (idx < items && row < R && n < nv) ? out[(size_t)row * ld + n] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kEpiBatch; ++u) {
+        const int idx = base + u * nthr;
+        if (idx >= items) break;   // warp-uniform (items and nthr are multiples of 32)
+        const int r = idx >> 7, v = idx & 127, row = r0 + r, n = v0 + v;
+        const bool ok = row < R && n < nv;
+        float y = tl[r * ldt + v];
+        if (scaled) y *= s_rs[r];
+        float hn = 0.f;
+        if (ok) {
+          hn = hres[u] + y;
+          out[(size_t)row * ld + n] = hn;
+          if (next_x)
+            store_act<T>(next_x, plane, (size_t)row * ld + n, hn * to_f32<T>(next_g[n]));
+        }
+        if (out_ss) {   // warp-uniform
+          const float sq = warp_sum(hn * hn);
+          float hw = 0.f;
+          if (head_w) {
+            const float gw = ok ? head_w[n] * to_f32<T>(next_g[n]) : 0.f;
+            hw = warp_sum(gw * hn);
+          }
+          if ((v & 31) == 0 && ok) {
+            out_ss[(size_t)(n >> 5) * ld_ss + row] = sq;
+            if (head_w) out_hw[(size_t)(n >> 5) * ld_ss + row] = hw;
+          }
+        }
+      }
+    }
   } else if (mode == EPI_SWIGLU) {
     T* const out_act = reinterpret_cast<T*>(a.out_act);
     const size_t ld_act = (size_t)a.ld_act, plane = (size_t)a.act_plane;
@@ -187,6 +275,50 @@ __device__ void tile_epilogue(const GemmArgs& a, int v0, int r0, int rt, const f
     const int layer = a.layer;
     const int hd = kv.hd, half = hd >> 1;
     const int nq = a.n_heads * hd, nk = kv.kvh * hd;
+    if constexpr (kBatch) if (qrows) {
+      const int items = rt * 128;
+      // kEpiBatch items per thread per pass: their RoPE factors in flight together
+      const size_t kv_pool = (size_t)kv.kvh * hd << kv.page_shift, h_pool = (size_t)hd
+                                                                             << kv.page_shift;
+      const size_t kv_tail = (size_t)kv.n_tail_slots * kv.kvh * hd, h_tail = (size_t)hd;
+      for (int base = tid; base < items; base += nthr * kEpiBatch) {
+        float2 cs[kEpiBatch];
+#pragma unroll
+        for (int u = 0; u < kEpiBatch; ++u) {
+          const int idx = base + u * nthr, row = r0 + (idx >> 7), n = v0 + (idx & 127);
+          cs[u] = (idx < items && row < R && n < nq + nk)
+                      ? rope[(size_t)qrows[row].pos * half + ((n % hd) % half)]
+                      : make_float2(1.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < kEpiBatch; ++u) {
+          const int idx = base + u * nthr, r = idx >> 7, v = idx & 127, row = r0 + r,
+                    n = v0 + v;
+          if (idx >= items || row >= R || n >= nq + 2 * nk) continue;
+          float y = tl[r * ldt + v];
+          if (scaled) y *= s_rs[r];
+          float val = y;
+          const int e = n % hd;
+          if (n < nq + nk) {
+            float other = (e < half) ? tl[r * ldt + v + half] : tl[r * ldt + v - half];
+            if (scaled) other *= s_rs[r];
+            val = (e < half) ? (y * cs[u].x - other * cs[u].y) : (y * cs[u].x + other * cs[u].y);
+          }
+          if (n < nq) {
+            q_out[(size_t)row * nq + n] = val;
+          } else {
+            const QkvRow m = qrows[row];
+            const int kvsel = (n < nq + nk) ? 0 : 1;
+            const int head = (n - nq - kvsel * nk) / hd;
+            if (m.where == 1)
+              kv.pool[(size_t)m.base + kvsel * kv_pool + head * h_pool + e] = val;
+            else if (m.where == 2)
+              kv.tail[(size_t)m.base + kvsel * kv_tail + head * h_tail + e] = val;
+          }
+        }
+      }
+      return;
+    }
     for (int idx = tid; idx < rt * 128; idx += nthr) {
       const int r = idx >> 7, v = idx & 127, row = r0 + r, n = v0 + v;
       if (row >= R || n >= nq + 2 * nk) continue;

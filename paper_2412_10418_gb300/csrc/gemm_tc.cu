@@ -78,7 +78,15 @@ __device__ __forceinline__ int unit_owner(int u, int U, int C) { return ((u + 1)
 
 constexpr int kMaxContrib = 256;   // contributors to one tile (bounded on the host)
 constexpr int kMaxSplit = 8;       // target blocks per tile when tiles are few
+constexpr int kRedBatch = 4;       // float4 groups per thread per pass of the large-row fixup
+constexpr int kBigRows = 64;       // padded activation rows above which k_gemm_tc<true> runs
 
+// kBig: the variant for more than 64 activation rows: its epilogue, stream-K fixup and
+// cluster reduction keep several loads per thread in flight (a tile's epilogue then costs a
+// few round trips to memory instead of one per row), and its QKV epilogue reads each row's
+// position and K/V destination gathered once per block. The plain loops of the other
+// variant keep its register count low, so that neighbouring launches overlap.
+template <bool kBig>
 __global__ void __launch_bounds__(kThreads, 1)
     k_gemm_tc(const __grid_constant__ TcMaps maps, const __grid_constant__ GemmArgs a, TcPlan p,
               float* part, int* tile_cnt) {
@@ -93,6 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ int s_abort, s_last;
   __shared__ int s_slot_off[kMaxContrib];   // reducer: scratch offset (floats) per contributor
   __shared__ float s_rs[256];                // input row scales (RMSNorm folded into the GEMM)
+  __shared__ QkvRow s_qkv[kBig ? 256 : 1];   // QKV: RoPE position and K/V destination per row
 
   uint8_t* smem = smem_raw + ((1024 - (tc::smem_u32(smem_raw) & 1023)) & 1023);
   const int NP = p.n_pad, S = p.stages, KBT = p.kb_total;
@@ -258,8 +267,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     int seg = 0;
     int u = u0;
     const int R = min(a.R, NP);
-    if (a.in_ss) {   // once per block, while the first accumulator fills
-      input_row_scales(a, 0, R, s_rs, etid, kEpThreads);
+    if (a.in_ss || (kBig && a.mode == EPI_QKV)) {   // once per block, while the first
+      if (a.in_ss) input_row_scales(a, 0, R, s_rs, etid, kEpThreads);   // accumulator fills
+      if (kBig && a.mode == EPI_QKV) qkv_rows(a, R, s_qkv, etid, kEpThreads);
       tc::named_barrier(1, kEpThreads);
     }
     while (u < u1) {
@@ -298,8 +308,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           // cluster split-K: the partial stays in tileS (ep_rows == NP: one chunk) until the
           // cluster reduction at the end
         } else if (whole) {
-          tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0, etid,
-                                       kEpThreads);
+          tile_epilogue<__nv_bfloat16, kBig>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0,
+                                             etid, kEpThreads, kBig ? s_qkv : nullptr);
+        } else if (kBig) {
+          for (int i = etid; i < rt * 32; i += kEpThreads) {   // float4 groups
+            const int r = i >> 5, v = (i & 31) * 4;
+            *reinterpret_cast<float4*>(my_part + (size_t)(r0 + r) * 128 + v) =
+                *reinterpret_cast<const float4*>(tileS + r * kTileLd + v);
+          }
         } else {
           for (int i = etid; i < rt * 128; i += kEpThreads) {
             const int r = i >> 7, v = i & 127;
@@ -329,30 +345,71 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int ncontrib = cl - cf + 1;
           for (int r0 = 0; r0 < R; r0 += kEpRows) {
             const int rt = min(kEpRows, R - r0);
-            // float4 groups: 32 per activation row; all contributors' loads in flight together
-            for (int i = etid; i < rt * 32; i += kEpThreads) {
-              const int off = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
-              float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-              int j = 0;
-              for (; j + 4 <= ncontrib; j += 4) {
-                float4 v[4];
+            if constexpr (kBig) {
+              // float4 groups, 32 per activation row, kRedBatch groups per thread per pass: the
+              // loads of kRedBatch groups x up to four contributors are in flight together. The
+              // contributors are summed in block order (deterministic).
+              for (int i0 = etid; i0 < rt * 32; i0 += kEpThreads * kRedBatch) {
+                float4 sum[kRedBatch];
+                int off[kRedBatch];
 #pragma unroll
-                for (int q = 0; q < 4; ++q)
-                  v[q] = __ldcg(reinterpret_cast<const float4*>(part + s_slot_off[j + q] + off));
+                for (int g = 0; g < kRedBatch; ++g) {
+                  const int i = min(i0 + g * kEpThreads, rt * 32 - 1);   // clamped: in bounds
+                  off[g] = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
+                  sum[g] = make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+                for (int j = 0; j < ncontrib; j += 4) {
+                  const int nj = min(4, ncontrib - j);
+                  float4 v[4][kRedBatch];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                  sum.x += v[q].x; sum.y += v[q].y; sum.z += v[q].z; sum.w += v[q].w;
+                  for (int q = 0; q < 4; ++q)
+#pragma unroll
+                    for (int g = 0; g < kRedBatch; ++g)
+                      if (q < nj)
+                        v[q][g] = __ldcg(
+                            reinterpret_cast<const float4*>(part + s_slot_off[j + q] + off[g]));
+#pragma unroll
+                  for (int q = 0; q < 4; ++q)
+#pragma unroll
+                    for (int g = 0; g < kRedBatch; ++g)
+                      if (q < nj) {
+                        sum[g].x += v[q][g].x; sum[g].y += v[q][g].y;
+                        sum[g].z += v[q][g].z; sum[g].w += v[q][g].w;
+                      }
+                }
+#pragma unroll
+                for (int g = 0; g < kRedBatch; ++g) {
+                  const int i = i0 + g * kEpThreads;
+                  if (i < rt * 32)
+                    *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum[g];
                 }
               }
-              for (; j < ncontrib; ++j) {
-                const float4 v = __ldcg(reinterpret_cast<const float4*>(part + s_slot_off[j] + off));
-                sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
+            } else {
+              // float4 groups: 32 per activation row; all contributors' loads in flight together
+              for (int i = etid; i < rt * 32; i += kEpThreads) {
+                const int off = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
+                float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+                int j = 0;
+                for (; j + 4 <= ncontrib; j += 4) {
+                  float4 v[4];
+#pragma unroll
+                  for (int q = 0; q < 4; ++q)
+                    v[q] = __ldcg(reinterpret_cast<const float4*>(part + s_slot_off[j + q] + off));
+#pragma unroll
+                  for (int q = 0; q < 4; ++q) {
+                    sum.x += v[q].x; sum.y += v[q].y; sum.z += v[q].z; sum.w += v[q].w;
+                  }
+                }
+                for (; j < ncontrib; ++j) {
+                  const float4 v = __ldcg(reinterpret_cast<const float4*>(part + s_slot_off[j] + off));
+                  sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
+                }
+                *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
               }
-              *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
             }
             tc::named_barrier(1, kEpThreads);
-            tile_epilogue<__nv_bfloat16>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0,
-                                         etid, kEpThreads);
+            tile_epilogue<__nv_bfloat16, kBig>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0,
+                                               etid, kEpThreads, kBig ? s_qkv : nullptr);
             tc::named_barrier(1, kEpThreads);
           }
           if (etid == 0) tile_cnt[t] = 0;
@@ -381,9 +438,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int i = etid; i < (rb - ra) * 32; i += kEpThreads) {
         const uint32_t off = ((ra + (i >> 5)) * kTileLd + (i & 31) * 4) * 4;
         float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int q = 0; q < SK; ++q) {
-          const float4 v = tc::ld_cluster_f32x4(tc::map_cluster_rank(tile_s + off, q));
-          sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
+        if constexpr (kBig) {
+          // eight blocks' loads in flight together, summed in rank order
+          for (int q0 = 0; q0 < SK; q0 += 8) {
+            float4 v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              if (q0 + q < SK)
+                v[q] = tc::ld_cluster_f32x4(tc::map_cluster_rank(tile_s + off, q0 + q));
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              if (q0 + q < SK) {
+                sum.x += v[q].x; sum.y += v[q].y; sum.z += v[q].z; sum.w += v[q].w;
+              }
+          }
+        } else {
+          for (int q = 0; q < SK; ++q) {
+            const float4 v = tc::ld_cluster_f32x4(tc::map_cluster_rank(tile_s + off, q));
+            sum.x += v.x; sum.y += v.y; sum.z += v.z; sum.w += v.w;
+          }
         }
         *reinterpret_cast<float4*>(red + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
       }
@@ -395,8 +468,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int etid = threadIdx.x - 64;
       tc::named_barrier(1, kEpThreads);
       if (rb > ra)
-        tile_epilogue<__nv_bfloat16>(a, t * 128, ra, rb - ra, red, kTileLd, s_rs + ra, etid,
-                                     kEpThreads);
+        tile_epilogue<__nv_bfloat16, kBig>(a, t * 128, ra, rb - ra, red, kTileLd, s_rs + ra,
+                                           etid, kEpThreads, kBig ? s_qkv : nullptr);
     }
     tc::cluster_wait();                 // no block leaves while its tile may still be read
   }
@@ -412,7 +485,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
-size_t g_static_smem = 4096;   // static shared memory of k_gemm_tc (queried at configuration)
+size_t g_static_smem[2] = {4096, 8192};   // static shared memory of k_gemm_tc<false / true>
+                                          // (queried at configuration)
 int g_max_cluster = 8;         // 16 where non-portable clusters of k_gemm_tc are allowed
 
 }  // namespace
@@ -434,15 +508,16 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   p.tiles = (n_virtual + 127) / 128;
   p.kb_total = K / 64;
   const size_t stage = 16384 + 256 * (size_t)p.n_pad;
+  p.big = p.n_pad > kBigRows;
   // two blocks per SM when three stages fit in half the shared memory (228 KB per SM, less
   // each block's static part and the 1 KB the runtime reserves per block), else one; the
   // epilogue drains 16 activation rows at a time when that frees room for another stage
-  const size_t half = 114 * 1024 - g_static_smem - 1024;
+  const size_t half = 114 * 1024 - g_static_smem[p.big] - 1024;
   auto fit = [&](size_t budget, int ep) {
     return (int)std::min<size_t>(kMaxStages, (budget - (size_t)ep * kTileLd * 4 - 1024) / stage);
   };
   int per_sm = 1;
-  size_t budget = 220 * 1024;
+  size_t budget = std::min<size_t>(220 * 1024, 227 * 1024 - g_static_smem[p.big]);
   const int ep_big = std::min(p.n_pad, kEpRowsMax);
   if (force_per_sm >= 3) {   // more, shallower blocks (measurement aid)
     per_sm = force_per_sm;
@@ -520,27 +595,39 @@ int encode_bf16_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t o
 }
 
 int configure_gemm_tc() {
-  cudaFuncAttributes fa;
-  if (cudaFuncGetAttributes(&fa, k_gemm_tc) != cudaSuccess) return -1;
-  g_static_smem = fa.sharedSizeBytes;
-  g_max_cluster =
-      cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess
-          ? 16
-          : 8;
-  cudaGetLastError();
-  return cudaFuncSetAttribute(k_gemm_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              220 * 1024 + 1024) == cudaSuccess
-             ? 0
-             : -1;
+  int rc = 0;
+  bool nonportable = true;
+  auto setup = [&](auto kernel, int big) {
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess) {
+      rc = -1;
+      return;
+    }
+    g_static_smem[big] = fa.sharedSizeBytes;
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+        cudaSuccess)
+      nonportable = false;
+    cudaGetLastError();
+    // plans use at most 220 KB + 1 KB of alignment slack; a block has at most 227 KB in all
+    const int dyn = (int)std::min<size_t>(220 * 1024 + 1024, 227 * 1024 - fa.sharedSizeBytes);
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn) !=
+        cudaSuccess)
+      rc = -1;
+  };
+  setup(k_gemm_tc<false>, 0);
+  setup(k_gemm_tc<true>, 1);
+  g_max_cluster = nonportable ? 16 : 8;
+  return rc;
 }
 
 void launch_gemm_tc(const TcMaps& maps, const GemmArgs& a, const TcPlan& p, float* part,
                     int* tile_cnt, cudaStream_t s) {
+  auto kernel = p.big ? k_gemm_tc<true> : k_gemm_tc<false>;
   if (p.cluster)
-    launch_pdl_cluster(k_gemm_tc, dim3(p.ctas), dim3(kThreads), p.smem, p.cluster, s, maps, a, p,
+    launch_pdl_cluster(kernel, dim3(p.ctas), dim3(kThreads), p.smem, p.cluster, s, maps, a, p,
                        part, tile_cnt);
   else
-    launch_pdl(k_gemm_tc, dim3(p.ctas), dim3(kThreads), p.smem, s, maps, a, p, part, tile_cnt);
+    launch_pdl(kernel, dim3(p.ctas), dim3(kThreads), p.smem, s, maps, a, p, part, tile_cnt);
 }
 
 }  // namespace cdsl

@@ -127,7 +127,8 @@ void launch_gemv(const GemmArgs& a, const GemvPlan& p, float* part, int* tile_cn
 struct TcMaps { CUtensorMap w[3]; CUtensorMap xh, xl; };
 // cluster > 0: cluster split-K with that many blocks per tile (ctas = tiles * cluster); 0:
 // persistent stream-K over ctas blocks.
-struct TcPlan { int tiles, kb_total, ctas, n_pad, stages, ep_rows, cluster; size_t smem; };
+// big: the variant for more than 64 activation rows (k_gemm_tc<true>)
+struct TcPlan { int tiles, kb_total, ctas, n_pad, stages, ep_rows, cluster, big; size_t smem; };
 bool tc_supported(const GemmArgs& a);
 // cluster: -1 chooses (split-K clusters when every tile fits at once with >= 2 blocks), 0
 // stream-K, > 0 that cluster size.
