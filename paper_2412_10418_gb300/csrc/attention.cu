@@ -341,9 +341,12 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
 }
 
 template <typename T, int HD, int QPW>
+ClusterFit g_fit;   // cluster residency of k_attn<T, HD, QPW> (configure_t)
+
+template <typename T, int HD, int QPW>
 void launch_t(const AttnArgs& a, int n_z, cudaStream_t s) {
-  const int cl = attn_cluster_size(g_max_cluster, a.n_chunks + a.n_tchunks, a.kv.kvh * n_z,
-                                   2 * kPlanSMs);
+  const int cl = attn_cluster_size(g_fit<T, HD, QPW>, g_max_cluster, a.n_chunks + a.n_tchunks,
+                                   a.kv.kvh * n_z);
   launch_pdl_cluster(k_attn<T, HD, QPW>, dim3(cl, a.kv.kvh, n_z), dim3(ATHREADS),
                      AttnSmem<HD>::bytes, cl, s, a);
 }
@@ -354,25 +357,11 @@ int configure_t() {
   if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AttnSmem<HD>::bytes) !=
       cudaSuccess)
     return -1;
-  if (cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
-    return 1;   // portable clusters only
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(ACL, 1, 1);
-  cfg.blockDim = dim3(ATHREADS);
-  cfg.dynamicSmemBytes = AttnSmem<HD>::bytes;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = ACL;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess || n < 1) {
-    cudaGetLastError();
-    return 1;
-  }
-  return 0;
+  const bool nonportable =
+      cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+  cudaGetLastError();
+  fill_cluster_fit(&g_fit<T, HD, QPW>, k, ATHREADS, AttnSmem<HD>::bytes, nonportable ? ACL : 8);
+  return nonportable && g_fit<T, HD, QPW>.active[ACL] >= 1 ? 0 : 1;   // 1: portable only
 }
 
 }  // namespace

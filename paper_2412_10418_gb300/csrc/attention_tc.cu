@@ -459,30 +459,19 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
 }
 
 template <int HD>
+ClusterFit g_tc_fit;   // cluster residency of k_attn_tc<HD> (configure_tc)
+
+template <int HD>
 int configure_tc() {
   auto k = k_attn_tc<HD>;
   if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)TcSmem<HD>::bytes) !=
       cudaSuccess)
     return -1;
-  if (cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
-    return 1;   // portable clusters only
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(TACL, 1, 1);
-  cfg.blockDim = dim3(TTHREADS);
-  cfg.dynamicSmemBytes = TcSmem<HD>::bytes;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = TACL;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess || n < 1) {
-    cudaGetLastError();
-    return 1;
-  }
-  return 0;
+  const bool nonportable =
+      cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+  cudaGetLastError();
+  fill_cluster_fit(&g_tc_fit<HD>, k, TTHREADS, TcSmem<HD>::bytes, nonportable ? TACL : 8);
+  return nonportable && g_tc_fit<HD>.active[TACL] >= 1 ? 0 : 1;   // 1: portable only
 }
 
 }  // namespace
@@ -504,8 +493,8 @@ int configure_attention_tc() {
 }
 
 void launch_attn_tc(const AttnArgs& a, int n_z, cudaStream_t s) {
-  const int cl = attn_cluster_size(g_tc_max_cluster, a.n_chunks + a.n_tchunks, a.kv.kvh * n_z,
-                                   kPlanSMs);
+  const int cl = attn_cluster_size(a.kv.hd == 128 ? g_tc_fit<128> : g_tc_fit<64>,
+                                   g_tc_max_cluster, a.n_chunks + a.n_tchunks, a.kv.kvh * n_z);
   if (a.kv.hd == 128)
     launch_pdl_cluster(k_attn_tc<128>, dim3(cl, a.kv.kvh, n_z), dim3(TTHREADS),
                        TcSmem<128>::bytes, cl, s, a);

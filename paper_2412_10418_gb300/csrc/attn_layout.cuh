@@ -179,17 +179,59 @@ __device__ void count_bytes(const Layout<QB>& L, const LaunchStamp& stamp, int q
 
 }  // namespace attn
 
+// Clusters of each size (1..16 blocks) that one attention kernel can keep resident at once
+// (cudaOccupancyMaxActiveClusters, queried at configuration; 0 where a size does not fit).
+struct ClusterFit {
+  int active[17] = {};
+};
+
+template <typename Kernel>
+void fill_cluster_fit(ClusterFit* f, Kernel kernel, int threads, size_t smem, int max_cluster) {
+  for (int c = 1; c <= max_cluster && c <= 16; ++c) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(c, 1, 1);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = c;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      n = 0;
+    }
+    f->active[c] = n;
+  }
+}
+
 // Blocks per cluster of an attention launch with `groups` clusters (prompt x KV head x query
-// block) over `chunks` key chunks, `slots` blocks resident at once: one chunk per block while
-// the groups leave room for that (the latency-bound decode and verify passes), fewer blocks
-// (more chunks each, in sequence) when the groups alone fill the GPU, so that a large pass
-// runs in about one wave instead of many waves of blocks that each do one chunk and merge.
-// A block takes at most attn::MAXCB chunks (its key-slot table), so the cluster never has
-// fewer than ceil(chunks / MAXCB) blocks (at most 8 for the 128 chunks of a pass).
-inline int attn_cluster_size(int max_cluster, int chunks, int groups, int slots) {
-  const int by_load = std::max(1, slots / std::max(1, groups));
-  const int least = (chunks + attn::MAXCB - 1) / attn::MAXCB;
-  return std::max(least, std::min(std::min(max_cluster, chunks), by_load));
+// block) over `chunks` key chunks: the size C with the least estimated time, waves(C) x
+// (2 ceil(chunks / C) + 1) in half chunk-times -- a block's chunks one after another, then
+// about half a chunk's time of merging -- where a wave is f.active[C] clusters. One chunk per
+// block while the groups leave room (the latency-bound decode and verify passes); fewer blocks
+// with more chunks each when one chunk per block would need more than a wave (a cluster too
+// large to be placed as often as the groups need it, e.g. 16 blocks, or too many groups). A
+// block takes at most attn::MAXCB chunks (its key-slot table), so C >= ceil(chunks / MAXCB);
+// ties go to the smaller cluster.
+inline int attn_cluster_size(const ClusterFit& f, int max_cluster, int chunks, int groups) {
+  const int least = std::max(1, (chunks + attn::MAXCB - 1) / attn::MAXCB);
+  const int most = std::max(least, std::min(std::min(max_cluster, 16), chunks));
+  int best = least;
+  long long best_cost = -1;
+  for (int c = least; c <= most; ++c) {
+    if (f.active[c] < 1) continue;
+    const long long waves = (groups + f.active[c] - 1) / f.active[c];
+    const long long cost = waves * (2LL * ((chunks + c - 1) / c) + 1);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = c;
+    }
+  }
+  return best;
 }
 
 }  // namespace cdsl
