@@ -77,7 +77,8 @@ struct cdsl_ctx {
   int32_t* lm_gather = nullptr;
   int32_t* lm_dst = nullptr;
   float* gemv_part = nullptr;   // split-K partial tiles of the weight-streaming GEMM
-  int32_t* gemv_cnt = nullptr;  // per-tile arrival counters
+  int32_t* gemv_cnt = nullptr;  // per-tile arrival counters, then per-tile finished shares
+  int plan_sms = kPlanSMs;      // SMs the tensor-core GEMM plans for: min(kPlanSMs, device's)
   int32_t* attn_zmap = nullptr; // prefill: z -> (prompt, query block)
   int attn_zmax = 0, attn_chunks = 0;
   StepState st{};
@@ -285,15 +286,17 @@ size_t carve(cdsl_ctx* c, void* base) {
         tiles = std::max(tiles, (size_t)p.tiles);
         if (c->dtype == CDSL_DTYPE_BF16 && sh[0] % 64 == 0) {
           for (int R = 9; R <= std::min(c->R_max, 256); R += 16) {  // every n_pad in use
+            // the plan, and stream-K, which a plan falls back to where clusters do not fit
             const TcPlan t = plan_tc(sh[0], sh[1], R, kPlanSMs);
-            part = std::max(part, tc_scratch_floats(t));
+            const TcPlan sk = plan_tc(sh[0], sh[1], R, kPlanSMs, 0, 0, 0);
+            part = std::max(part, std::max(tc_scratch_floats(t), tc_scratch_floats(sk)));
             tiles = std::max(tiles, (size_t)t.tiles);
           }
         }
       }
     }
     c->gemv_part = cv.take<float>(part);
-    c->gemv_cnt = cv.take<int32_t>(tiles);
+    c->gemv_cnt = cv.take<int32_t>(2 * tiles);
   }
   {  // attention: the prefill's (prompt, query block) map
     const int QB = attn_qblock();
@@ -419,7 +422,7 @@ void gemm(cdsl_ctx* c, const GemmArgs& a) {
       maps.w[s] = tensor_map(c, a.w[seg], a.K, a.seg_rows[seg], 64);
     }
     const __nv_bfloat16* xb = reinterpret_cast<const __nv_bfloat16*>(a.x);
-    const TcPlan p = plan_tc(a.K, a.n_virtual, a.R, kPlanSMs);
+    const TcPlan p = plan_tc(a.K, a.n_virtual, a.R, c->plan_sms);
     // activation boxes: 64 features x n_pad rows (<= 256 <= R_pad), one per plane and stage
     maps.xh = tensor_map(c, xb, a.ldx, c->R_pad, p.n_pad);
     maps.xl = tensor_map(c, xb + a.x_plane, a.ldx, c->R_pad, p.n_pad);
@@ -787,6 +790,12 @@ int32_t cdsl_init(const cdsl_model_cfg* target, const void* const* h_target_weig
   if (c->dtype == CDSL_DTYPE_BF16 && configure_gemm_tc()) {
     delete c;
     return fail(nullptr, CDSL_ECUDA, "cannot configure the tensor-core GEMM (shared memory)");
+  }
+  {  // the large-row GEMM's stream-K grid must be resident at once (one block per SM)
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && sms > 0)
+      c->plan_sms = std::min(kPlanSMs, sms);
   }
   cudaMemsetAsync(d_workspace, 0, c->ws_total, c->stream);
   launch_rope_table(c->tgt.rope, c->lrope, target->head_dim, target->rope_theta, c->stream);

@@ -179,35 +179,6 @@ __device__ void count_bytes(const Layout<QB>& L, const LaunchStamp& stamp, int q
 
 }  // namespace attn
 
-// Clusters of each size (1..16 blocks) that one attention kernel can keep resident at once
-// (cudaOccupancyMaxActiveClusters, queried at configuration; 0 where a size does not fit).
-struct ClusterFit {
-  int active[17] = {};
-};
-
-template <typename Kernel>
-void fill_cluster_fit(ClusterFit* f, Kernel kernel, int threads, size_t smem, int max_cluster) {
-  for (int c = 1; c <= max_cluster && c <= 16; ++c) {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(c, 1, 1);
-    cfg.blockDim = dim3(threads);
-    cfg.dynamicSmemBytes = smem;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = c;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
-      cudaGetLastError();
-      n = 0;
-    }
-    f->active[c] = n;
-  }
-}
-
 // Blocks per cluster of an attention launch with `groups` clusters (prompt x KV head x query
 // block) over `chunks` key chunks: the size C with the least estimated time, waves(C) x
 // (2 ceil(chunks / C) + 1) in half chunk-times -- a block's chunks one after another, then

@@ -102,6 +102,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ int s_slot_off[kMaxContrib];   // reducer: scratch offset (floats) per contributor
   __shared__ float s_rs[256];                // input row scales (RMSNorm folded into the GEMM)
   __shared__ QkvRow s_qkv[kBig ? 256 : 1];   // QKV: RoPE position and K/V destination per row
+  __shared__ int s_pend[2], s_npend;         // kBig stream-K: tiles this block helps finish
 
   uint8_t* smem = smem_raw + ((1024 - (tc::smem_u32(smem_raw) & 1023)) & 1023);
   const int NP = p.n_pad, S = p.stages, KBT = p.kb_total;
@@ -160,6 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc::mbar_init(&drain_bar, 1);
     s_abort = 0;
+    s_npend = 0;
     tc::fence_mbar_init();
     tc::fence_proxy_async();
     // the first ring's weights do not depend on the previous kernel: issue them while warp 1
@@ -330,61 +332,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int cf = unit_owner(t * KBT, U, C);
         const int cl = unit_owner((t + 1) * KBT - 1, U, C);
         // publish this block's partial and count it (one acquire-release atomic after the
-        // barrier; the last block to arrive then sees every contributor's partial)
+        // barrier)
         tc::named_barrier(1, kEpThreads);
-        if (etid == 0) s_last = (tc::atom_add_acq_rel_gpu(tile_cnt + t, 1) == cl - cf);
-        tc::named_barrier(1, kEpThreads);
-        if (s_last) {
-          // scratch slot of every contributor: its first segment -> 0, its last -> 1
-          for (int j = etid; j <= cl - cf; j += kEpThreads) {
-            const int cc = cf + j;
-            const int sl = (t == unit_start(cc, U, C) / KBT) ? 0 : 1;
-            s_slot_off[j] = (cc * 2 + sl) * NP * 128;
+        if constexpr (kBig) {
+          // the tile is finished after this block's last segment, by all its contributors
+          if (etid == 0) {
+            tc::atom_add_acq_rel_gpu(tile_cnt + t, 1);
+            s_pend[s_npend++] = t;
           }
+        } else {
+          // the last block to arrive sees every contributor's partial and finishes the tile
+          if (etid == 0) s_last = (tc::atom_add_acq_rel_gpu(tile_cnt + t, 1) == cl - cf);
           tc::named_barrier(1, kEpThreads);
-          const int ncontrib = cl - cf + 1;
-          for (int r0 = 0; r0 < R; r0 += kEpRows) {
-            const int rt = min(kEpRows, R - r0);
-            if constexpr (kBig) {
-              // float4 groups, 32 per activation row, kRedBatch groups per thread per pass: the
-              // loads of kRedBatch groups x up to four contributors are in flight together. The
-              // contributors are summed in block order (deterministic).
-              for (int i0 = etid; i0 < rt * 32; i0 += kEpThreads * kRedBatch) {
-                float4 sum[kRedBatch];
-                int off[kRedBatch];
-#pragma unroll
-                for (int g = 0; g < kRedBatch; ++g) {
-                  const int i = min(i0 + g * kEpThreads, rt * 32 - 1);   // clamped: in bounds
-                  off[g] = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
-                  sum[g] = make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-                for (int j = 0; j < ncontrib; j += 4) {
-                  const int nj = min(4, ncontrib - j);
-                  float4 v[4][kRedBatch];
-#pragma unroll
-                  for (int q = 0; q < 4; ++q)
-#pragma unroll
-                    for (int g = 0; g < kRedBatch; ++g)
-                      if (q < nj)
-                        v[q][g] = __ldcg(
-                            reinterpret_cast<const float4*>(part + s_slot_off[j + q] + off[g]));
-#pragma unroll
-                  for (int q = 0; q < 4; ++q)
-#pragma unroll
-                    for (int g = 0; g < kRedBatch; ++g)
-                      if (q < nj) {
-                        sum[g].x += v[q][g].x; sum[g].y += v[q][g].y;
-                        sum[g].z += v[q][g].z; sum[g].w += v[q][g].w;
-                      }
-                }
-#pragma unroll
-                for (int g = 0; g < kRedBatch; ++g) {
-                  const int i = i0 + g * kEpThreads;
-                  if (i < rt * 32)
-                    *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum[g];
-                }
-              }
-            } else {
+          if (s_last) {
+            // scratch slot of every contributor: its first segment -> 0, its last -> 1
+            for (int j = etid; j <= cl - cf; j += kEpThreads) {
+              const int cc = cf + j;
+              const int sl = (t == unit_start(cc, U, C) / KBT) ? 0 : 1;
+              s_slot_off[j] = (cc * 2 + sl) * NP * 128;
+            }
+            tc::named_barrier(1, kEpThreads);
+            const int ncontrib = cl - cf + 1;
+            for (int r0 = 0; r0 < R; r0 += kEpRows) {
+              const int rt = min(kEpRows, R - r0);
               // float4 groups: 32 per activation row; all contributors' loads in flight together
               for (int i = etid; i < rt * 32; i += kEpThreads) {
                 const int off = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
@@ -406,17 +376,97 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum;
               }
+              tc::named_barrier(1, kEpThreads);
+              tile_epilogue<__nv_bfloat16, false>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0,
+                                                  etid, kEpThreads);
+              tc::named_barrier(1, kEpThreads);
             }
-            tc::named_barrier(1, kEpThreads);
-            tile_epilogue<__nv_bfloat16, kBig>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0,
-                                               etid, kEpThreads, kBig ? s_qkv : nullptr);
-            tc::named_barrier(1, kEpThreads);
+            if (etid == 0) tile_cnt[t] = 0;
           }
-          if (etid == 0) tile_cnt[t] = 0;
         }
       }
       u = seg_end;
       ++seg;
+    }
+    if constexpr (kBig) {
+      // Distributed stream-K fixup: every contributor of a partially owned tile sums its share
+      // of the tile's activation rows over all contributors' partials (block order, as the
+      // single-finisher form would) and runs the epilogue on them, once every partial of the
+      // tile is published. Each block publishes all its partials before it waits, and every
+      // block of the grid is resident at once (one block per SM, no more blocks than SMs), so
+      // every wait ends; it is still bounded. tile_cnt[tiles + t] counts the finished shares;
+      // the last one resets both counters for the next launch.
+      const bool gave_up = tc::named_barrier_or(1, kEpThreads, s_abort != 0);
+      const int npend = gave_up ? 0 : s_npend;
+      for (int q = 0; q < npend; ++q) {
+        const int t = s_pend[q];
+        const int cf = unit_owner(t * KBT, U, C);
+        const int cl = unit_owner((t + 1) * KBT - 1, U, C);
+        const int ncontrib = cl - cf + 1, jme = c - cf;
+        bool ok = true;
+        if (etid == 0) ok = tc::wait_count_gpu(tile_cnt + t, ncontrib, a.status, a.wait_ns);
+        if (tc::named_barrier_or(1, kEpThreads, !ok)) {
+          s_abort = 1;
+          break;
+        }
+        // scratch slot of every contributor: its first segment -> 0, its last -> 1
+        for (int j = etid; j < ncontrib; j += kEpThreads) {
+          const int cc = cf + j;
+          const int sl = (t == unit_start(cc, U, C) / KBT) ? 0 : 1;
+          s_slot_off[j] = (cc * 2 + sl) * NP * 128;
+        }
+        tc::named_barrier(1, kEpThreads);
+        const int ra = jme * R / ncontrib, rb = (jme + 1) * R / ncontrib;
+        for (int rs = ra; rs < rb; rs += kEpRows) {
+          const int rt = min(kEpRows, rb - rs), r0 = rs;
+          // float4 groups, 32 per activation row, kRedBatch groups per thread per pass: the
+          // loads of kRedBatch groups x up to four contributors are in flight together. The
+          // contributors are summed in block order (deterministic).
+          for (int i0 = etid; i0 < rt * 32; i0 += kEpThreads * kRedBatch) {
+            float4 sum[kRedBatch];
+            int off[kRedBatch];
+#pragma unroll
+            for (int g = 0; g < kRedBatch; ++g) {
+              const int i = min(i0 + g * kEpThreads, rt * 32 - 1);   // clamped: in bounds
+              off[g] = (r0 + (i >> 5)) * 128 + (i & 31) * 4;
+              sum[g] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            for (int j = 0; j < ncontrib; j += 4) {
+              const int nj = min(4, ncontrib - j);
+              float4 v[4][kRedBatch];
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int g = 0; g < kRedBatch; ++g)
+                  if (q < nj)
+                    v[q][g] = __ldcg(
+                        reinterpret_cast<const float4*>(part + s_slot_off[j + q] + off[g]));
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+#pragma unroll
+                for (int g = 0; g < kRedBatch; ++g)
+                  if (q < nj) {
+                    sum[g].x += v[q][g].x; sum[g].y += v[q][g].y;
+                    sum[g].z += v[q][g].z; sum[g].w += v[q][g].w;
+                  }
+            }
+#pragma unroll
+            for (int g = 0; g < kRedBatch; ++g) {
+              const int i = i0 + g * kEpThreads;
+              if (i < rt * 32)
+                *reinterpret_cast<float4*>(tileS + (i >> 5) * kTileLd + (i & 31) * 4) = sum[g];
+            }
+          }
+          tc::named_barrier(1, kEpThreads);
+          tile_epilogue<__nv_bfloat16, true>(a, t * 128, r0, rt, tileS, kTileLd, s_rs + r0, etid,
+                                             kEpThreads, s_qkv);
+          tc::named_barrier(1, kEpThreads);
+        }
+        if (etid == 0 && tc::atom_add_acq_rel_gpu(tile_cnt + p.tiles + t, 1) == ncontrib - 1) {
+          tile_cnt[t] = 0;
+          tile_cnt[p.tiles + t] = 0;
+        }
+      }
     }
   }
   if (SK > 0) {
@@ -488,6 +538,11 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 size_t g_static_smem[2] = {4096, 8192};   // static shared memory of k_gemm_tc<false / true>
                                           // (queried at configuration)
 int g_max_cluster = 8;         // 16 where non-portable clusters of k_gemm_tc are allowed
+// Clusters of k_gemm_tc<big> resident at once with one or two blocks' shared memory budget per
+// SM ([big][blocks per SM - 1]; configure_gemm_tc fills [1][0], the one in use; until then no
+// plan is limited).
+ClusterFit g_cfit[2][2];
+bool g_cfit_ready = false;
 
 }  // namespace
 
@@ -519,7 +574,8 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
   int per_sm = 1;
   size_t budget = std::min<size_t>(220 * 1024, 227 * 1024 - g_static_smem[p.big]);
   const int ep_big = std::min(p.n_pad, kEpRowsMax);
-  if (force_per_sm >= 3) {   // more, shallower blocks (measurement aid)
+  if (force_per_sm >= 3 && !p.big) {   // more, shallower blocks (measurement aid; the
+                                         // large-row variant's fixup needs one block per SM)
     per_sm = force_per_sm;
     budget = (227 * 1024) / force_per_sm - 1024;
   } else if ((force_per_sm == 2 || force_per_sm == 0) && fit(half, 16) >= 3) {
@@ -549,6 +605,13 @@ TcPlan plan_tc(int K, int n_virtual, int R, int n_sm, int force_per_sm, int max_
             ? std::max(std::min(8, cap / p.tiles), std::min(12, wide / p.tiles))
             : 0;
   S = std::min(std::min(S, p.kb_total), g_max_cluster);
+  // large-row plans (one block per SM): every cluster must be resident at once. A cluster is
+  // placed whole within a GPC, so fewer clusters fit than the SMs suggest (g_cfit: e.g. the
+  // small model's 18-tile QKV at 160 rows, 7-block clusters: 42.9 -> 28.2 us with 6). The
+  // reported residency at two blocks per SM is below what the 7B plans measurably get
+  // (limiting them by it: 7B step 5.95 -> 7.10 ms), so those keep the measured caps above.
+  if (g_cfit_ready && p.big && per_sm == 1)
+    while (S >= 2 && g_cfit[1][0].active[S] < p.tiles) --S;
   if (S >= 2 && tile_fits) {
     p.cluster = S;
     p.ctas = p.tiles * S;
@@ -617,6 +680,11 @@ int configure_gemm_tc() {
   setup(k_gemm_tc<false>, 0);
   setup(k_gemm_tc<true>, 1);
   g_max_cluster = nonportable ? 16 : 8;
+  if (rc == 0) {
+    const size_t one = std::min<size_t>(220 * 1024 + 1024, 227 * 1024 - g_static_smem[1]);
+    fill_cluster_fit(&g_cfit[1][0], k_gemm_tc<true>, kThreads, one, g_max_cluster);
+    g_cfit_ready = true;
+  }
   return rc;
 }
 

@@ -114,6 +114,35 @@ void launch_gemm_simt(int dtype, const GemmArgs& a, cudaStream_t s);
 // Weight-streaming GEMM for R <= 8 activation rows (bf16 weights), split-K over `splits`
 // slices of k_split elements. Scratch: part [splits][8][tiles][128] floats and one arrival
 // counter per tile (zero between launches).
+// Clusters of each size (1..16 blocks) that one kernel can keep resident at once
+// (cudaOccupancyMaxActiveClusters, queried at configuration; 0 where a size does not fit).
+struct ClusterFit {
+  int active[17] = {};
+};
+
+template <typename Kernel>
+void fill_cluster_fit(ClusterFit* f, Kernel kernel, int threads, size_t smem, int max_cluster) {
+  for (int c = 1; c <= max_cluster && c <= 16; ++c) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(c, 1, 1);
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = c;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      n = 0;
+    }
+    f->active[c] = n;
+  }
+}
+
 struct GemvPlan { int splits, k_split, tiles; };
 constexpr int kPlanSMs = 152;  // GB300: split-K is planned for this many SMs
 GemvPlan plan_gemv(int K, int n_virtual, int n_sm);

@@ -132,6 +132,28 @@ __device__ __forceinline__ int atom_add_acq_rel_gpu(int* p, int v) {
   return old;
 }
 
+// Wait until *p >= n (acquire at GPU scope: the writes published before the increments that
+// reached n are then visible to this thread, and to its block after a barrier). False (and
+// CDSL_ETIMEOUT latched in *status) if that has not happened after limit_ns.
+__device__ __forceinline__ bool wait_count_gpu(const int* p, int n, int32_t* status,
+                                               uint64_t limit_ns) {
+  auto load = [&]() {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+  };
+  if (load() >= n) return true;
+  const uint64_t t0 = globaltimer();
+  while (load() < n) {
+    if (globaltimer() - t0 > limit_ns) {
+      set_status(status, CDSL_ETIMEOUT);
+      return false;
+    }
+    __nanosleep(100);
+  }
+  return true;
+}
+
 // ------------------------------------------------------------------------------ TMA
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
