@@ -66,8 +66,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   const int C = (int)gridDim.x;                 // = cluster size
   const int cx = (int)blockIdx.x;               // = rank in the cluster
   const int g = blockIdx.y;
-  const int n_p = a.n_chunks, NC = a.n_chunks + a.n_tchunks;
-  const int nb_chunks = (NC - cx + C - 1) / C;  // this block's chunks cx, cx + C, ...
+  const int n_p = a.n_chunks;
   int b, qb;
   if (a.zmap) {
     b = a.zmap[2 * blockIdx.z];
@@ -82,7 +81,8 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   // ---- this cluster's query vectors and this block's key slots. The rows (plan kernel), the
   //      committed page table and the tail layout come from kernels the launch chain has
   //      already completed, so all of it precedes the wait.
-  const int nq = attn::build_layout<QB, ATHREADS>(L, a, b, qb, cx, C, nb_chunks);
+  const int nq = attn::build_layout<QB, ATHREADS>(L, a, b, qb, cx, C);
+  const int nb_chunks = L.nb;                     // chunk_of(L, n_p, cx, C, 0 .. nb_chunks - 1)
   const int maxnp = L.maxnp;
   if (a.stamp) attn::count_bytes<QB, ATHREADS, HD>(L, stamp, qb, cx, nb_chunks, nq, &s_nkeys);
   pdl_wait();                 // q and K/V of the previous kernels are ready
@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(ATHREADS, 2) k_attn(AttnArgs a) {
   }
   bool q_staged = false;
   for (int i = 0; i < nb_chunks && nq > 0; ++i) {
-    const int c = cx + i * C;
+    const int c = attn::chunk_of(L, n_p, cx, C, i);
     const bool tail = c >= n_p;
     const int t0 = c * ACH;
     if (!tail && t0 >= maxnp) continue;   // beyond every query vector's prefix

@@ -17,10 +17,12 @@
 // transposed as the P V product's B operand). Q is split once per block, pre-scaled by
 // 1/sqrt(head_dim).
 //
-// Softmax: warp w < 4 reads TMEM lanes 32w..32w+31, so each of its threads owns one query
-// vector's row of scores (no shuffles). The running reference m is raised only when a chunk's
+// Softmax: warps w and w + 4 read TMEM lanes 32(w % 4) .. +31, so each thread owns one query
+// vector's row of scores over half the chunk's keys (the two halves exchange their row
+// maxima through shared memory; each keeps its own share of the row sum). The running reference m is raised only when a chunk's
 // maximum exceeds it by more than kLazy (then O in TMEM and l are rescaled); otherwise
-// p = exp(s - m) <= e^kLazy, and the final o / l does not depend on the reference. The
+// p = exp(s - m) <= e^8, and the final o / l does not depend on the reference. Scores are kept
+// in base 2 (q is pre-scaled by log2(e) / sqrt(head_dim), p = 2^(s - m)). The
 // block's partial (m, l, o) are merged across the cluster through distributed shared memory
 // as in attention.cu, and the normalized output is written as the O projection's hi/lo input.
 //
@@ -48,7 +50,9 @@ constexpr int TTHREADS = 256;
 constexpr int TWARPS = TTHREADS / 32;
 constexpr int TACL = 16;             // blocks per cluster (at most)
 constexpr int kIssuer = 128;         // thread that issues the MMAs (warp 4, lane 0)
-constexpr float kLazy = 8.0f;        // raise the softmax reference only past this margin
+constexpr float kLazy = 11.5415602f; // raise the softmax reference only past this margin
+                                     // (base-2 scores: 8 / ln 2, so p <= e^8)
+constexpr float kLog2e = 1.44269504088896341f;
 
 int g_tc_max_cluster = 8;
 
@@ -110,19 +114,20 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
   __shared__ int s_abort, s_nkeys;
   __shared__ const float* s_kptr[ACH];            // K of each key slot of the chunk (V follows)
   __shared__ float s_pm[TQB], s_pl[TQB];          // the block's partial (m, l) per query vector
+  __shared__ float s_mx[2][TQB];                  // per half: a chunk's row maxima, then l
 
   cg::cluster_group cluster = cg::this_cluster();
   const int C = (int)gridDim.x;                   // = cluster size
   const int cx = (int)blockIdx.x;                 // = rank in the cluster
   const int g = blockIdx.y;
-  const int n_p = a.n_chunks, NC = a.n_chunks + a.n_tchunks;
-  const int nb_chunks = (NC - cx + C - 1) / C;    // this block's chunks cx, cx + C, ...
+  const int n_p = a.n_chunks;
   const int b = blockIdx.z / a.qb_count, qb = blockIdx.z % a.qb_count;
   const int G = a.G, H = a.n_heads;
   const int warp = threadIdx.x >> 5;
 
   // ---- query vectors and key slots (before the wait: inputs of completed kernels only)
-  const int nq = attn::build_layout<TQB, TTHREADS>(L, a, b, qb, cx, C, nb_chunks);
+  const int nq = attn::build_layout<TQB, TTHREADS>(L, a, b, qb, cx, C);
+  const int nb_chunks = L.nb;                     // chunk_of(L, n_p, cx, C, 0 .. nb_chunks - 1)
   const int maxnp = L.maxnp;
   if (a.stamp) attn::count_bytes<TQB, TTHREADS, HD>(L, stamp, qb, cx, nb_chunks, nq, &s_nkeys);
   if (threadIdx.x == 0) {
@@ -146,13 +151,14 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
   const uint32_t idesc_s = tc::idesc_bf16_f32(128, ACH), idesc_o = tc::idesc_bf16_f32(128, HD);
   const size_t v_delta_tail = (size_t)a.kv.n_tail_slots * a.kv.kvh * HD;
   const size_t v_delta_pfx = ((size_t)a.kv.kvh << a.kv.page_shift) * HD;
-  const int qi = threadIdx.x;                      // softmax threads (warps 0-3): TMEM lane
+  const int qi = threadIdx.x & (TQB - 1);          // softmax: TMEM lane (query vector) and
+  const int half = threadIdx.x / TQB;              //   half of the chunk's keys
   float m_ref = -INFINITY, l_run = 0.f;
   int nproc = 0;                                    // chunks whose P V has been issued
   bool q_staged = false;
 
   for (int i = 0; i < nb_chunks && nq > 0; ++i) {
-    const int c = cx + i * C;
+    const int c = attn::chunk_of(L, n_p, cx, C, i);
     const bool tail = c >= n_p;
     const int t0 = c * ACH;
     if (!tail && t0 >= maxnp) continue;             // beyond every query vector's prefix
@@ -212,7 +218,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
 #pragma unroll
       for (int u = 0; u < Q_IT; ++u) {
         const int it = threadIdx.x + u * TTHREADS, qv = it / DCH, dc = it % DCH;
-        const float sc = a.scale;
+        const float sc = a.scale * kLog2e;   // base-2 scores
         const float x[8] = {qr[u][0].x * sc, qr[u][0].y * sc, qr[u][0].z * sc, qr[u][0].w * sc,
                             qr[u][1].x * sc, qr[u][1].y * sc, qr[u][1].z * sc, qr[u][1].w * sc};
         uint4 hi, lo;
@@ -263,84 +269,89 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
       }
       tc::umma_commit(&bar_s);
     }
-    // ---- softmax over the chunk: thread qi owns TMEM lane qi (a query vector's 64 scores)
-    if (warp < 4) {
-      // the whole warp takes the same branch (tcgen05.ld is warp-collective)
-      if (!__all_sync(0xffffffffu, tc::mbar_wait(&bar_s, nproc & 1, a.status, a.wait_ns))) {
-        s_abort = 1;
-      } else {
-        tc::tc_fence_after();
-        float s[4][16];
-        {
-          uint32_t r[4][16];
+    // ---- softmax over the chunk: thread t owns TMEM lane qi = t % 128 (a query vector) and
+    //      the chunk's keys 32h .. 32h + 31, h = t / 128 (warps w and w + 4 read the same
+    //      lanes; tcgen05.ld is warp-collective, so a warp takes every branch as a whole)
+    const bool sok = __all_sync(0xffffffffu, tc::mbar_wait(&bar_s, nproc & 1, a.status, a.wait_ns));
+    float s[2][16];
+    float mx = -INFINITY;
+    if (!sok) {
+      s_abort = 1;
+    } else {
+      tc::tc_fence_after();
+      uint32_t r[2][16];
 #pragma unroll
-          for (int q = 0; q < 4; ++q) tc::tmem_ld16_nowait(t_s + lane_base + 16 * q, r[q]);
-          tc::tmem_wait_ld();
+      for (int q = 0; q < 2; ++q)
+        tc::tmem_ld16_nowait(t_s + lane_base + 32 * half + 16 * q, r[q]);
+      tc::tmem_wait_ld();
+      // prefix chunk: key j is visible below the row's prefix length (one limit per row)
+      const int lim = (!tail && qi < nq) ? L.np[qi] - t0 - 32 * half : 0;
 #pragma unroll
-          for (int q = 0; q < 4; ++q)
+      for (int q = 0; q < 2; ++q)
 #pragma unroll
-            for (int e = 0; e < 16; ++e) s[q][e] = __uint_as_float(r[q][e]);
+        for (int e = 0; e < 16; ++e) {
+          const int j = 32 * half + 16 * q + e;
+          const bool vis = tail ? (qi < nq && attn::key_visible(L, qi, i, c, n_p, j))
+                                : 16 * q + e < lim;
+          s[q][e] = vis ? __uint_as_float(r[q][e]) : -INFINITY;   // masked: 2^(-inf - m) = 0
+          mx = fmaxf(mx, s[q][e]);
         }
-        float mx = -INFINITY;
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            const int j = 16 * q + e;
-            const bool vis = qi < nq && attn::key_visible(L, qi, i, c, n_p, j);
-            s[q][e] = vis ? s[q][e] : -INFINITY;   // masked keys: exp(-inf - m) = 0 below
-            mx = fmaxf(mx, s[q][e]);
-          }
-        // raise the reference where a row's maximum passed it by more than kLazy: its earlier
-        // sum and output are rescaled by alpha = exp(m_old - m_new)
-        float alpha = 1.f;
-        bool rescale_o = false;
-        if (mx > -INFINITY && (m_ref == -INFINITY || mx > m_ref + kLazy)) {
-          alpha = m_ref == -INFINITY ? 0.f : expf(m_ref - mx);
-          rescale_o = nproc > 0 && m_ref > -INFINITY;
-          l_run *= alpha;
-          m_ref = mx;
-        }
-        // the output rows in TMEM are rescaled by the whole warp (tcgen05.ld / st are
-        // warp-collective), each lane by its own factor (1 where its reference stayed)
-        if (__any_sync(0xffffffffu, rescale_o)) {
-          const float f = rescale_o ? alpha : 1.f;
-#pragma unroll 1
-          for (int q = 0; q < HD / 16; ++q) {
-            float o[16];
-            tc::tmem_ld16(t_o + lane_base + 16 * q, o);
-#pragma unroll
-            for (int e = 0; e < 16; ++e) o[e] *= f;
-            tc::tmem_st16(t_o + lane_base + 16 * q, o);
-          }
-        }
-        float sum = 0.f;
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-#pragma unroll
-          for (int e = 0; e < 16; ++e) {
-            s[q][e] = m_ref == -INFINITY ? 0.f : expf(s[q][e] - m_ref);
-            sum += s[q][e];
-          }
-        l_run += sum;
-        // P row qi: keys 8ch..8ch+7 are 16-byte chunk ch (hi and lo planes)
-#pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-          float x[8];
-#pragma unroll
-          for (int e = 0; e < 8; ++e) x[e] = s[ch >> 1][(ch & 1) * 8 + e];
-          uint4 hi, lo;
-          split8(x, hi, lo);
-          const uint32_t off = SM::P_OFF + tc::sw128_offset(qi, ch);
-          st_shared16(sm, off, hi);
-          st_shared16(sm, off + SM::P_PLANE, lo);
-        }
-        tc::fence_proxy_async();
-      }
-      tc::tc_fence_before();
+      s_mx[half][qi] = mx;
     }
     __syncthreads();
     if (s_abort) break;
+    mx = fmaxf(s_mx[0][qi], s_mx[1][qi]);   // the row's maximum, the same in both halves
+    {
+      // raise the reference where a row's maximum passed it by more than kLazy: its earlier
+      // sum and output are rescaled by alpha = exp(m_old - m_new) (both halves decide alike)
+      float alpha = 1.f;
+      bool rescale_o = false;
+      if (mx > -INFINITY && (m_ref == -INFINITY || mx > m_ref + kLazy)) {
+        alpha = m_ref == -INFINITY ? 0.f : exp2f(m_ref - mx);
+        rescale_o = nproc > 0 && m_ref > -INFINITY;
+        l_run *= alpha;
+        m_ref = mx;
+      }
+      // each half rescales its half of the output row's columns, each lane by its own factor
+      // (1 where its reference stayed)
+      if (__any_sync(0xffffffffu, rescale_o)) {
+        const float f = rescale_o ? alpha : 1.f;
+#pragma unroll 1
+        for (int q = 0; q < HD / 32; ++q) {
+          float o[16];
+          const uint32_t col = t_o + lane_base + half * (HD / 2) + 16 * q;
+          tc::tmem_ld16(col, o);
+#pragma unroll
+          for (int e = 0; e < 16; ++e) o[e] *= f;
+          tc::tmem_st16(col, o);
+        }
+      }
+      float sum = 0.f;
+#pragma unroll
+      for (int q = 0; q < 2; ++q)
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          s[q][e] = m_ref == -INFINITY ? 0.f : exp2f(s[q][e] - m_ref);
+          sum += s[q][e];
+        }
+      l_run += sum;   // this half's share of the row's sum; the halves are added at the end
+      // P row qi: keys 8ch..8ch+7 are 16-byte chunk ch (hi and lo planes); this half writes
+      // chunks 4h .. 4h + 3
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        float x[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) x[e] = s[cc >> 1][(cc & 1) * 8 + e];
+        uint4 hi, lo;
+        split8(x, hi, lo);
+        const uint32_t off = SM::P_OFF + tc::sw128_offset(qi, 4 * half + cc);
+        st_shared16(sm, off, hi);
+        st_shared16(sm, off + SM::P_PLANE, lo);
+      }
+      tc::fence_proxy_async();
+      tc::tc_fence_before();
+    }
+    __syncthreads();
     // ---- O += P V (hi.hi + hi.lo + lo.hi over the chunk's 64 keys)
     if (threadIdx.x == kIssuer) {
       tc::tc_fence_after();
@@ -365,43 +376,45 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
     tc::umma_commit(&bar_d);
     tc::mbar_wait(&bar_d, 0, a.status);
   }
-  // ---- the block's partial (m, l, o) per query vector into shared memory (o over K, V, P)
-  if (warp < 4 && nproc > 0 && !tc::mbar_wait(&bar_o, (nproc - 1) & 1, a.status, a.wait_ns))
-    s_abort = 1;
+  // ---- the block's partial (m, l, o) per query vector into shared memory (o over K, V, P):
+  //      each half writes its half of the row's columns; l is the sum of the halves' shares
+  if (nproc > 0 && !tc::mbar_wait(&bar_o, (nproc - 1) & 1, a.status, a.wait_ns)) s_abort = 1;
+  if (half == 1) s_mx[1][qi] = l_run;
   __syncthreads();
   float* s_po = reinterpret_cast<float*>(sm + SM::O_OFF);   // [TQB][OP]
   const bool have_o = nproc > 0 && !s_abort;
-  if (warp < 4) {
-    if (have_o) tc::tc_fence_after();
+  if (have_o) tc::tc_fence_after();
 #pragma unroll 1
-    for (int q0 = 0; q0 < HD / 16; q0 += 4) {   // 64 columns per wait
-      uint32_t o[4][16];
+  for (int q0 = 0; q0 < HD / 32; q0 += 4) {   // 64 columns per wait
+    uint32_t o[4][16];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        if (have_o) {
-          tc::tmem_ld16_nowait(t_o + lane_base + 16 * (q0 + q), o[q]);
-        } else {
+    for (int q = 0; q < 4; ++q) {
+      if (have_o && q0 + q < HD / 32) {
+        tc::tmem_ld16_nowait(t_o + lane_base + half * (HD / 2) + 16 * (q0 + q), o[q]);
+      } else {
 #pragma unroll
-          for (int e = 0; e < 16; ++e) o[q][e] = 0u;
-        }
+        for (int e = 0; e < 16; ++e) o[q][e] = 0u;
       }
-      if (have_o) tc::tmem_wait_ld();
-      if (qi < nq) {
+    }
+    if (have_o) tc::tmem_wait_ld();
+    if (qi < nq) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q)
+      for (int q = 0; q < 4; ++q)
+        if (q0 + q < HD / 32)
 #pragma unroll
-          for (int e = 0; e < 16; e += 4)
-            *reinterpret_cast<float4*>(s_po + qi * SM::OP + 16 * (q0 + q) + e) =
+          for (int e = 0; e < 16; e += 4) {
+            float* dst = s_po + qi * SM::OP + half * (HD / 2) + 16 * (q0 + q) + e;
+            *reinterpret_cast<float4*>(dst) =
                 make_float4(__uint_as_float(o[q][e]), __uint_as_float(o[q][e + 1]),
                             __uint_as_float(o[q][e + 2]), __uint_as_float(o[q][e + 3]));
-      }
+          }
     }
-    if (qi < nq) {
-      s_pm[qi] = have_o ? m_ref : -INFINITY;
-      s_pl[qi] = have_o ? l_run : 0.f;
-    }
-    tc::tc_fence_before();
   }
+  if (half == 0 && qi < nq) {
+    s_pm[qi] = have_o ? m_ref : -INFINITY;
+    s_pl[qi] = have_o ? l_run + s_mx[1][qi] : 0.f;
+  }
+  tc::tc_fence_before();
   cluster.sync();   // every block's partials are visible to the cluster
 
   // ---- merge: block cx finishes query vectors cx, cx + C, ... (a warp per query vector),
@@ -434,7 +447,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
       lr = cluster.map_shared_rank(s_pl, lane)[qv];
     }
     const float M = warp_max(mr);
-    const float w = (lane < C && mr > -INFINITY) ? expf(mr - M) : 0.f;
+    const float w = (lane < C && mr > -INFINITY) ? exp2f(mr - M) : 0.f;
     const float Lsum = warp_sum(w * lr);
     float acc[DPL];
 #pragma unroll

@@ -5,7 +5,11 @@
 // chunks of ACH slots: prefix chunks (ACH consecutive positions of the prompt's shared prefix
 // pages) and then tail chunks (the distinct beam tails of a query block's rows, concatenated,
 // each as long as its longest row). A cluster of blocks owns one (prompt b, KV head, query
-// block qb); block cx of the C blocks takes chunks cx, cx + C, ... A query vector is a (row,
+// block qb). The launch sizes for the most chunks a pass can have (n_chunks prefix chunks,
+// n_tchunks tail chunks); the chunks that hold keys -- prefix chunks below the block's longest
+// prefix, tail chunks up to the tails' total length -- are numbered in order, and block cx of
+// the C blocks takes numbers cx, cx + C, ..., so the cluster's work is spread evenly over
+// the chunks that exist at run time. A query vector is a (row,
 // query head of the KV head's GQA group) pair; the rows of prompt b are taken in row order,
 // G vectors each, and query block qb holds vectors [qb * QB, qb * QB + QB).
 #pragma once
@@ -32,22 +36,30 @@ struct Layout {
                                      // tail's offset in the concatenation, length, base slot
   int wcnt[32];                      // scratch: rows of prompt b per warp
   int nrows, maxnp;                  // rows of prompt b seen so far; longest prefix
+  int nr_p, nr_t, nb;                // prefix and tail chunks holding keys; this block's chunks
   int kslot[MAXCB * ACH];            // every key slot of the block's chunks: the page (prefix
                                      // chunk) or tail row (tail chunk), -1 empty
   int ktb[MAXCB * ACH];              // tail slots: tail base of the beam,
   uint8_t kj[MAXCB * ACH];           //   index in it
 };
 
-// Fill L for query block qb of prompt b and this block's chunks (cx, cx + C, ..., nb_chunks of
-// them); called by all NTHREADS threads of the block (a multiple of 32, at most 1024), which
-// it leaves synchronized. Reads only what the launch chain has already completed (row
+// Pass chunk (prefix chunks first, n_p of them) of this block's i-th chunk: number cx + i * C
+// among the chunks that hold keys (L.nr_p prefix, then L.nr_t tail chunks).
+template <int QB>
+__device__ __forceinline__ int chunk_of(const Layout<QB>& L, int n_p, int cx, int C, int i) {
+  const int k = cx + i * C;
+  return k < L.nr_p ? k : n_p + (k - L.nr_p);
+}
+
+// Fill L for query block qb of prompt b and this block's chunks (L.nb of them, chunk_of);
+// called by all NTHREADS threads of the block (a multiple of 32, at most 1024), which it
+// leaves synchronized. Reads only what the launch chain has already completed (row
 // descriptors, committed page table), so it may run before griddepcontrol.wait. Returns the
 // number of the block's query vectors (0..a.qblock). At most 32 rows may meet in one query block
 // (the tail layout runs one lane per row). More tail keys than the tail chunks hold latch
 // CDSL_ERANGE.
 template <int QB, int NTHREADS>
-__device__ int build_layout(Layout<QB>& L, const AttnArgs& a, int b, int qb, int cx, int C,
-                            int nb_chunks) {
+__device__ int build_layout(Layout<QB>& L, const AttnArgs& a, int b, int qb, int cx, int C) {
   constexpr int NWARPS = NTHREADS / 32;
   const int G = a.G, QBr = a.qblock;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -121,13 +133,16 @@ __device__ int build_layout(Layout<QB>& L, const AttnArgs& a, int b, int qb, int
     if (lane == 0) {
       L.maxnp = np;
       if (cx == 0 && total > a.n_tchunks * ACH) set_status(a.status, CDSL_ERANGE);
+      L.nr_p = min(a.n_chunks, (np + ACH - 1) / ACH);
+      L.nr_t = min(a.n_tchunks, (total + ACH - 1) / ACH);
+      L.nb = max(0, (L.nr_p + L.nr_t - cx + C - 1) / C);   // <= MAXCB: C >= chunks / MAXCB
     }
   }
   __syncthreads();
-  const int maxnp = L.maxnp, n_p = a.n_chunks;
+  const int maxnp = L.maxnp, n_p = a.n_chunks, nb_chunks = L.nb;
   // key slots of this block's chunks
   for (int i = 0; i < nb_chunks; ++i) {
-    const int c = cx + i * C;
+    const int c = chunk_of(L, n_p, cx, C, i);
     if (c < n_p) {   // prefix positions c*ACH .. c*ACH + ACH-1 below the longest prefix
       for (int j = threadIdx.x; j < ACH; j += NTHREADS) {
         const int t = c * ACH + j;
