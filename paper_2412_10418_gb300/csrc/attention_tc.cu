@@ -112,7 +112,8 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
   __shared__ __align__(8) uint64_t bar_d;          // every MMA of the block has completed
   __shared__ uint32_t s_tmem;
   __shared__ int s_abort, s_nkeys;
-  __shared__ const float* s_kptr[ACH];            // K of each key slot of the chunk (V follows)
+  __shared__ const float* s_kptr[2][ACH];         // K of each key slot of a chunk (V follows);
+                                                  // chunk i uses buffer i & 1
   __shared__ float s_pm[TQB], s_pl[TQB];          // the block's partial (m, l) per query vector
   __shared__ float s_mx[2][TQB];                  // per half: a chunk's row maxima, then l
 
@@ -128,7 +129,6 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
   // ---- query vectors and key slots (before the wait: inputs of completed kernels only)
   const int nq = attn::build_layout<TQB, TTHREADS>(L, a, b, qb, cx, C);
   const int nb_chunks = L.nb;                     // chunk_of(L, n_p, cx, C, 0 .. nb_chunks - 1)
-  const int maxnp = L.maxnp;
   if (a.stamp) attn::count_bytes<TQB, TTHREADS, HD>(L, stamp, qb, cx, nb_chunks, nq, &s_nkeys);
   if (threadIdx.x == 0) {
     tc::mbar_init(&bar_s, 1);
@@ -155,50 +155,32 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
   const int half = threadIdx.x / TQB;              //   half of the chunk's keys
   float m_ref = -INFINITY, l_run = 0.f;
   int nproc = 0;                                    // chunks whose P V has been issued
-  bool q_staged = false;
 
-  for (int i = 0; i < nb_chunks && nq > 0; ++i) {
-    const int c = attn::chunk_of(L, n_p, cx, C, i);
-    const bool tail = c >= n_p;
-    const int t0 = c * ACH;
-    if (!tail && t0 >= maxnp) continue;             // beyond every query vector's prefix
-    // the previous chunk's P V has completed: K, V and P may be overwritten
-    if (nproc > 0 && !tc::mbar_wait(&bar_o, (nproc - 1) & 1, a.status, a.wait_ns)) s_abort = 1;
+  // Staging is software-pipelined: chunk i + 1's K and V rows are loaded from the fp32 cache
+  // into registers right after chunk i's score MMAs are issued (in flight during its
+  // softmax), and converted and stored once chunk i's P V has completed.
+  auto kptrs = [&](int i) {   // threads 0 .. ACH-1: key slot pointers of chunk i
     if (threadIdx.x < ACH) {
+      const int c = attn::chunk_of(L, n_p, cx, C, i);
       const int ks = L.kslot[i * ACH + threadIdx.x];
       const float* kp = nullptr;
-      if (ks >= 0)
-        kp = tail ? a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, ks, g)
-                  : a.kv.pool + kv_prefix_offset(a.kv, a.layer, ks, 0, g,
-                                                 (t0 + threadIdx.x) & ((1 << a.kv.page_shift) - 1));
-      s_kptr[threadIdx.x] = kp;
-    }
-    __syncthreads();
-    if (s_abort) break;
-    // ---- stage the chunk (and Q with the first one): all loads in flight together, then
-    //      split and store. Q: query vector qi is row qi of the A operand (zero rows from nq
-    //      on), pre-scaled by 1/sqrt(head_dim).
-    const size_t v_delta = tail ? v_delta_tail : v_delta_pfx;
-    float4 qr[Q_IT][2];
-    float4 kr[K_IT][2];
-    float vr[V_IT][8];
-    if (!q_staged) {
-#pragma unroll
-      for (int u = 0; u < Q_IT; ++u) {
-        const int it = threadIdx.x + u * TTHREADS, qv = it / DCH, dc = it % DCH;
-        qr[u][0] = qr[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (qv < nq) {
-          const float* src =
-              a.q + (size_t)L.row[qv] * H * HD + (size_t)(g * G + L.gg[qv]) * HD + dc * 8;
-          qr[u][0] = *reinterpret_cast<const float4*>(src);
-          qr[u][1] = *reinterpret_cast<const float4*>(src + 4);
-        }
+      if (ks >= 0) {
+        const int slot = (c * ACH + threadIdx.x) & ((1 << a.kv.page_shift) - 1);
+        kp = c >= n_p ? a.kv.tail + kv_tail_offset(a.kv, a.layer, 0, ks, g)
+                      : a.kv.pool + kv_prefix_offset(a.kv, a.layer, ks, 0, g, slot);
       }
+      s_kptr[i & 1][threadIdx.x] = kp;
     }
+  };
+  float4 kr[K_IT][2];   // raw K and V of the next chunk to stage
+  float vr[V_IT][8];
+  auto load_kv = [&](int i) {   // all loads of chunk i in flight together (pointers ready)
+    const size_t v_delta = attn::chunk_of(L, n_p, cx, C, i) >= n_p ? v_delta_tail : v_delta_pfx;
+    const float* const* kps = s_kptr[i & 1];
 #pragma unroll
     for (int u = 0; u < K_IT; ++u) {
       const int idx = threadIdx.x + u * TTHREADS, j = idx / DCH, dc = idx % DCH;
-      const float* kp = s_kptr[j];
+      const float* kp = kps[j];
       kr[u][0] = kr[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
       if (kp) {
         kr[u][0] = __ldg(reinterpret_cast<const float4*>(kp + dc * 8));
@@ -210,25 +192,51 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
       const int idx = threadIdx.x + u * TTHREADS, d = idx % HD, jc = idx / HD;
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
-        const float* kp = s_kptr[jc * 8 + q];
+        const float* kp = kps[jc * 8 + q];
         vr[u][q] = kp ? __ldg(kp + v_delta + d) : 0.f;
       }
     }
-    if (!q_staged) {
+  };
+  if (nb_chunks > 0 && nq > 0) {
+    // ---- Q once per block: query vector qi is row qi of the A operand (zero rows from nq
+    //      on), pre-scaled by log2(e) / sqrt(head_dim) (base-2 scores); and chunk 0's loads
+    kptrs(0);
+    float4 qr[Q_IT][2];
 #pragma unroll
-      for (int u = 0; u < Q_IT; ++u) {
-        const int it = threadIdx.x + u * TTHREADS, qv = it / DCH, dc = it % DCH;
-        const float sc = a.scale * kLog2e;   // base-2 scores
-        const float x[8] = {qr[u][0].x * sc, qr[u][0].y * sc, qr[u][0].z * sc, qr[u][0].w * sc,
-                            qr[u][1].x * sc, qr[u][1].y * sc, qr[u][1].z * sc, qr[u][1].w * sc};
-        uint4 hi, lo;
-        split8(x, hi, lo);
-        const uint32_t off = SM::Q_OFF + (dc >> 3) * SM::Q_KB + tc::sw128_offset(qv, dc & 7);
-        st_shared16(sm, off, hi);
-        st_shared16(sm, off + SM::Q_PLANE, lo);
+    for (int u = 0; u < Q_IT; ++u) {
+      const int it = threadIdx.x + u * TTHREADS, qv = it / DCH, dc = it % DCH;
+      qr[u][0] = qr[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (qv < nq) {
+        const float* src =
+            a.q + (size_t)L.row[qv] * H * HD + (size_t)(g * G + L.gg[qv]) * HD + dc * 8;
+        qr[u][0] = *reinterpret_cast<const float4*>(src);
+        qr[u][1] = *reinterpret_cast<const float4*>(src + 4);
       }
-      q_staged = true;
     }
+    __syncthreads();   // chunk 0's pointers
+    load_kv(0);
+#pragma unroll
+    for (int u = 0; u < Q_IT; ++u) {
+      const int it = threadIdx.x + u * TTHREADS, qv = it / DCH, dc = it % DCH;
+      const float sc = a.scale * kLog2e;
+      const float x[8] = {qr[u][0].x * sc, qr[u][0].y * sc, qr[u][0].z * sc, qr[u][0].w * sc,
+                          qr[u][1].x * sc, qr[u][1].y * sc, qr[u][1].z * sc, qr[u][1].w * sc};
+      uint4 hi, lo;
+      split8(x, hi, lo);
+      const uint32_t off = SM::Q_OFF + (dc >> 3) * SM::Q_KB + tc::sw128_offset(qv, dc & 7);
+      st_shared16(sm, off, hi);
+      st_shared16(sm, off + SM::Q_PLANE, lo);
+    }
+  }
+
+  for (int i = 0; i < nb_chunks && nq > 0; ++i) {
+    const int c = attn::chunk_of(L, n_p, cx, C, i);
+    const bool tail = c >= n_p;
+    const int t0 = c * ACH;
+    // the previous chunk's P V has completed: K, V and P may be overwritten
+    if (nproc > 0 && !tc::mbar_wait(&bar_o, (nproc - 1) & 1, a.status, a.wait_ns)) s_abort = 1;
+    if (i + 1 < nb_chunks) kptrs(i + 1);
+    // ---- stage the chunk: split the loaded K and V into hi/lo and store
 #pragma unroll
     for (int u = 0; u < K_IT; ++u) {
       const int idx = threadIdx.x + u * TTHREADS, j = idx / DCH, dc = idx % DCH;
@@ -251,6 +259,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
     }
     tc::fence_proxy_async();
     __syncthreads();
+    if (s_abort) break;
     // ---- S = Q K^T (hi.hi + hi.lo + lo.hi over the head dimension)
     if (threadIdx.x == kIssuer) {
       tc::tc_fence_after();
@@ -269,6 +278,7 @@ __global__ void __launch_bounds__(TTHREADS, 1) k_attn_tc(AttnArgs a) {
       }
       tc::umma_commit(&bar_s);
     }
+    if (i + 1 < nb_chunks) load_kv(i + 1);   // in flight during this chunk's softmax
     // ---- softmax over the chunk: thread t owns TMEM lane qi = t % 128 (a query vector) and
     //      the chunk's keys 32h .. 32h + 31, h = t / 128 (warps w and w + 4 read the same
     //      lanes; tcgen05.ld is warp-collective, so a warp takes every branch as a whole)
