@@ -61,13 +61,26 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* m, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// The same test with a suspend-time hint: a thread whose phase is not complete yet sleeps
+// until it completes or about 2 us pass, instead of spinning (7B step 5.825 -> 5.813 ms).
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* m, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(m)), "r"(parity), "r"(2000u)
+      : "memory");
+  return ok != 0;
+}
 // Wait for the phase of parity `parity` to complete; false (and CDSL_ETIMEOUT latched in
 // *status) if it has not after limit_ns.
 __device__ __forceinline__ bool mbar_wait(uint64_t* m, uint32_t parity, int32_t* status,
                                           uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(m, parity)) return true;
   const uint64_t t0 = globaltimer();
-  while (!mbar_try_wait(m, parity)) {
+  while (!mbar_try_wait_sleep(m, parity)) {
     if (globaltimer() - t0 > limit_ns) {
       set_status(status, CDSL_ETIMEOUT);
       return false;
