@@ -90,7 +90,7 @@ typedef struct cdsl_run_cfg {
   float r_t;            /* reward threshold */
   int32_t reward_head;  /* 0: R = coverage; 1: R = 0.5 coverage + 0.5 sigmoid(w . h_last) */
   int32_t page_size;    /* KV page size in tokens (power of two, 16..256); 0 = 64 */
-  int32_t max_chunk;    /* rows per prefill forward pass; 0 = 64 */
+  int32_t max_chunk;    /* rows per prefill forward pass; 0 = 256 (the tensor-core GEMM maximum) */
   /* Validation of the lookahead by M_p (Sec. 3.2.2):
    *   0: hard rejection: x_j is accepted while argmax p_j == x_j;
    *   1: speculative sampling: x_j is accepted while u_j <= min(1, p_j(x_j) / q_j(x_j)),

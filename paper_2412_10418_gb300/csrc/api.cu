@@ -214,9 +214,10 @@ void derive_dims(cdsl_ctx* c) {
   c->R_d = c->B * c->k + c->B;
   // Step-1 round 2: the target pass holds d+2 rows per prompt (draft calls fit in R_d)
   c->R_s1 = r.step1_budget >= 2 ? c->B * (c->d + 2) : 0;
-  // default 64 prefill rows: the projections then stay on the fused hi/lo MMA with two blocks
-  // per SM (measured: 54 ms for the 512-token 7B prefill, against 96 ms at 256 rows)
-  const int chunk = r.max_chunk ? r.max_chunk : 64;
+  // default 256 prefill rows (the most the tensor-core GEMM takes): the large-row GEMM then
+  // streams each weight once per 256 prompt tokens (measured, 512-token 7B prefill: 43 ms at
+  // 64 rows, 35 at 128, 33 at 256; 13B, 4 x 1024 tokens: 564, 464, 428 ms)
+  const int chunk = r.max_chunk ? r.max_chunk : 256;
   c->R_p = std::min(chunk, c->B * r.max_prompt);
   c->R_max = std::max(std::max(c->R_v, c->R_s1), std::max(c->R_d, c->R_p));
   c->R_pad = (c->R_max + 31) / 32 * 32;

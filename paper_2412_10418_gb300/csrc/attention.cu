@@ -5,9 +5,9 @@
 // into chunks of 64 slots: prefix chunks of 64 consecutive prefix positions, then tail chunks
 // holding the distinct beam tails of a query block's rows (each row masked to its own beam and
 // causal within it). A thread-block cluster of up to 16 blocks owns one prompt, one KV head
-// and one query block of 16 or 32 query vectors (query vector = (row, query head of the GQA
-// group)); block r of the cluster takes chunks r, r + C, ... (one chunk each while the pass
-// has at most 16). For each chunk it loads K and V once into shared memory and scores all its
+// and one query block of 16, 32 or 40 query vectors (query vector = (row, query head of the
+// GQA group)); the chunks that hold keys are dealt to the cluster's blocks in turn (one chunk
+// each while the pass has no more chunks than blocks; attn_layout.cuh). For each chunk it loads K and V once into shared memory and scores all its
 // query vectors against them, keeping a running (max m, sum of exponentials l, unnormalized
 // output o) per query vector (split-KV with an online softmax, fp32). The cluster then merges
 // its blocks' partials through distributed shared memory, each block finishing a share of the

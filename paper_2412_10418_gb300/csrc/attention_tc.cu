@@ -2,10 +2,10 @@
 // 5th-generation tensor cores (tcgen05 MMA into TMEM).
 //
 // The pass is split as in attention.cu (attn_layout.cuh): a thread-block cluster of up to 16
-// blocks owns one (prompt, KV head, query block) and block cx of it the key chunks cx, cx + C,
-// ... (64 key slots each: prefix positions, then the query block's beam tails). A query block
-// holds up to 128 query vectors -- the MMA's M -- so the 7B verify pass (80 query vectors per
-// KV head) is one block per chunk and KV head.
+// blocks owns one (prompt, KV head, query block), and the chunks of 64 key slots that hold
+// keys (prefix positions, then the query block's beam tails) are dealt to its blocks in turn.
+// A query block holds up to 128 query vectors -- the MMA's M -- so the 7B verify pass (80
+// query vectors per KV head) is one block per chunk and KV head.
 //
 // Per chunk, with every operand a K-major bf16 tile in 128-byte-swizzled shared memory:
 //   S = Q K^T      M = 128 query vectors, N = 64 keys, K = head_dim  -> TMEM columns [0, 64)
@@ -13,18 +13,20 @@
 // fp32 accuracy from bf16 operands: every fp32 input x is split into hi = bf16(x) and
 // lo = bf16(x - hi), and each product is hi.hi + hi.lo + lo.hi (lo.lo, about 2^-18 of the
 // product, is dropped), accumulated in fp32. The K/V cache stays fp32 in HBM; the block
-// converts its chunk while staging it (K row-major as the score product's B operand, V
-// transposed as the P V product's B operand). Q is split once per block, pre-scaled by
-// 1/sqrt(head_dim).
+// converts each chunk while staging it (K row-major as the score product's B operand, V
+// transposed as the P V product's B operand). Staging is software-pipelined: the next
+// chunk's rows are loaded into registers while this chunk's softmax runs and stored once
+// its P V has completed. Q is split once per block, pre-scaled by log2(e) / sqrt(head_dim)
+// (scores in base 2).
 //
 // Softmax: warps w and w + 4 read TMEM lanes 32(w % 4) .. +31, so each thread owns one query
 // vector's row of scores over half the chunk's keys (the two halves exchange their row
-// maxima through shared memory; each keeps its own share of the row sum). The running reference m is raised only when a chunk's
-// maximum exceeds it by more than kLazy (then O in TMEM and l are rescaled); otherwise
-// p = exp(s - m) <= e^8, and the final o / l does not depend on the reference. Scores are kept
-// in base 2 (q is pre-scaled by log2(e) / sqrt(head_dim), p = 2^(s - m)). The
-// block's partial (m, l, o) are merged across the cluster through distributed shared memory
-// as in attention.cu, and the normalized output is written as the O projection's hi/lo input.
+// maxima through shared memory; each keeps its own share of the row sum). The running
+// reference m is raised only when a chunk's maximum exceeds it by more than kLazy (then O in
+// TMEM and l are rescaled); otherwise p = 2^(s - m) <= e^8, and the final o / l does not
+// depend on the reference. The block's partial (m, l, o) are merged across the cluster
+// through distributed shared memory as in attention.cu, and the normalized output is written
+// as the O projection's hi/lo input.
 //
 // One thread issues every MMA; tcgen05.commit arrives on an mbarrier that the consumers wait
 // on (bounded by the launch's wait limit: on expiry CDSL_ETIMEOUT is latched and the block

@@ -15,10 +15,11 @@
 // streams weights and activations with TMA through a ring of mbarrier-guarded stages; warp 1
 // (one lane) issues the MMAs into one of two TMEM accumulators and commits; warps 2-5 drain a
 // finished accumulator (TMEM -> registers -> shared memory) while the next segment
-// accumulates into the other one. A segment covering a
-// whole tile runs the fused epilogue directly; otherwise its partial tile goes to scratch and
-// the last contributing block of that tile adds the partials in block order (a deterministic
-// sum) and runs the epilogue.
+// accumulates into the other one. A segment covering a whole tile runs the fused epilogue
+// directly; otherwise its partial tile goes to scratch and the tile is finished from the
+// partials summed in block order (a deterministic sum): by the last contributing block
+// (k_gemm_tc<false>), or above 64 activation rows (k_gemm_tc<true>) by every contributor for
+// its share of the rows, after its own last segment, once all partials are in.
 //
 // Cluster split-K (GEMMs with few tiles): a thread-block cluster of S blocks owns one tile and
 // block r of it the r-th of S even K ranges. Each block drains its partial tile into shared
