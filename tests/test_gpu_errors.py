@@ -82,3 +82,28 @@ def test_expired_waits_latch_etimeout_and_the_device_stays_usable():
     eng2, states, rep, adopted, n = run_parity(s, steps=3, tol=2e-2, tol_r=2e-2)
     assert n == 3 and eng2.status() == cdsl.CDSL_OK
     eng2.close()
+
+
+def test_expired_waits_in_the_large_row_gemm_and_tensor_core_attention():
+    """The same with k = 8, d = 8: 72 verify rows, so the projections run the large-row GEMM
+    (more than 64 rows: stream-K with the contributors' shared fixup, whose counter waits are
+    bounded too) and the verify attention runs on the tensor cores (72 query vectors per KV
+    head). Every block gives up or finishes, the launches end, and a new context on the same
+    device matches the oracle at this shape."""
+    import torch
+    import paper_2412_10418_gb300 as cdsl
+    from cdsl_parity import run_parity
+
+    s = make_setup(synth.scaled(synth.SMALL, batch=1, k=8, d=8, max_new=8))
+    eng = engine(s)
+    eng.step()
+    assert eng.status() == cdsl.CDSL_OK
+    cdsl.cdsl_set_wait_limit(eng.ctx, 0)
+    eng.step()
+    assert eng.status() == cdsl.CDSL_ETIMEOUT
+    torch.cuda.synchronize()
+    eng.close()
+
+    eng2, states, rep, adopted, n = run_parity(s, steps=2, tol=2e-2, tol_r=2e-2)
+    assert n == 2 and eng2.status() == cdsl.CDSL_OK
+    eng2.close()
