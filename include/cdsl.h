@@ -259,11 +259,10 @@ CDSL_API int32_t cdsl_get_status(cdsl_ctx* ctx, int32_t* h_device_status);
  * the hi/lo activation planes, 8.3 MiB) is one fixed array inside the library, which every
  * GPU that loads the library holds until the process exits; no call allocates or frees.
  * Set-up: the first call in each CUDA context looks up that array's device address (and
- * clears its counters) with the context current, so make that first call before any stream
- * capture. Only contexts that stay alive are supported: after a device reset the array's
- * address may be stale. Every call shares the array: calls that overlap on a GPU (other
- * streams or threads) race, and the caller must order them. Asynchronous on `stream`;
- * errors via cdsl_last_error(NULL). */
+ * clears its counters) with the context current. Only contexts that stay alive are
+ * supported: after a device reset the array's address may be stale. Every call shares the
+ * array: calls that overlap on a GPU (other streams or threads) race, and the caller must
+ * order them. Asynchronous on `stream`; errors via cdsl_last_error(NULL). */
 CDSL_API int32_t cdsl_gemv_noalloc(const void* d_w, int32_t N, int32_t K, const float* d_x,
                                    int32_t R, float* d_y, void* stream);
 
